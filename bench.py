@@ -1,0 +1,436 @@
+#!/usr/bin/env python3
+"""Benchmark of the absorbed-MLA decode step on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+
+Prints ONE JSON line (rank 0).  A step is one pass of the whole decode path
+over one batch: cache append of this step's q_len entries, query absorption,
+split-KV attention over the latent cache, split combine, W_UV (and W_O)
+projection.  `value` is latent-cache throughput in GB/s (cache bytes the step
+must read / step time) with every input resident in HBM; the step replays as a
+CUDA graph and rotates over enough replicas of the inputs that the bytes
+touched between two reuses exceed twice the L2.  `roofline` rates the
+attention kernel (the dominant one) on its own launches, timed with CUDA
+events on its stream.  `e2e` repeats the step through the public API with the
+step's inputs copied from pinned host memory and the output read back.
+`cpu_baseline` (rank 0, N = 1) times the fp64 CPU oracle on a bounded sample.
+
+Under torchrun (N > 1) every rank runs its own replica of the workload on its
+own GPU (weak scaling, no collective on the data path); the timing is the
+maximum over ranks and `value` sums the bytes of all ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+DEFAULT_WORKLOAD = "qwen05b_b16_h14_r256_t2048"
+METRIC = "MLA decode-attn μs/step and latent-cache HBM GB/s (% of GB300 peak), 1 GPU"
+
+
+def parse_args(argv=None):
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--num-splits", type=int, default=0)
+    p.add_argument("--no-graph", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--seed", type=int, default=0)
+    return p.parse_args(argv)
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def max_over_ranks(value: float, world: int, device=None) -> float:
+    """Largest value over all ranks (the slowest rank sets the job's time)."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(value: float, world: int, device=None) -> float:
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ---------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 200 ms in the background."""
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+        self.t0 = self.t1 = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(prefix="clocks_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (FileNotFoundError, OSError):
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or not self.path or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = []
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[4:9]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        names = ["active_mask", "hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, r in rows for i in range(1, 5) if r[i].lower().startswith("active")})
+        sm = sorted(x[0] for x in rows)
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(x[1] for x in rows), "reasons": reasons,
+                "samples": len(rows)}
+
+
+# ---------------------------------------------------------------- our arm
+
+def run_ours(args, rank, world, local):
+    import torch
+    from paper_2607_27269_gb300 import abi
+    from paper_2607_27269_gb300 import workloads as wl
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    abi.lib()
+    shape = wl.SHAPES[args.workload]
+    w = wl.make(shape, seed=args.seed + rank)
+    cache_bytes = w.cache_bytes
+    props = torch.cuda.get_device_properties(dev)
+    l2 = getattr(props, "L2_cache_size", 126 * 2 ** 20)
+    # bytes one step touches: the cache it reads plus the query / weight / output tensors
+    per_replica = (w.c_kv.numel() + w.k_rope.numel()) * 2 + sum(
+        t.numel() * t.element_size() for t in (w.w_uk, w.w_uv, w.q_nope, w.q_pe, w.c_new, w.kr_new)
+        if t is not None) + (w.w_o.numel() * 2 if w.w_o is not None else 0)
+    replicas = max(2, math.ceil(2 * l2 / per_replica) + 1)
+    dws = [abi.to_device(w, dev) for _ in range(replicas)]
+    steps = [abi.DecodeStep(d.dims, d.cache, d.batch, d.q_len, d.max_kv_len, args.num_splits) for d in dws]
+    S = steps[0].num_splits
+
+    def run(i):
+        d, st = dws[i % replicas], steps[i % replicas]
+        return st(d.q_nope, d.q_pe, d.kv_len, d.w_uk, d.w_uv, d.w_o, c_new=d.c_new, kr_new=d.kr_new,
+                  start_pos=d.start_pos)
+
+    stream = torch.cuda.Stream(dev)
+    with torch.cuda.stream(stream):
+        for i in range(max(args.warmup, 3)):
+            run(i)
+        code = abi.check_status(stream)
+        if code != abi.MLA_OK:
+            raise RuntimeError(f"device status after warm-up: {abi.status_name(code)}")
+
+        graphs = None
+        if not args.no_graph:
+            graphs = []
+            for i in range(replicas):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=stream):
+                    run(i)
+                graphs.append(g)
+            for i in range(replicas):
+                graphs[i].replay()
+        torch.cuda.synchronize(dev)
+
+        def one(i):
+            if graphs is not None:
+                graphs[i % replicas].replay()
+            else:
+                run(i)
+
+        # ---- timed region: exactly K steps
+        clocks = ClockSampler(local)
+        clocks.start()
+        barrier(world)
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(args.steps):
+            one(i)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        barrier(world)
+        elapsed_ms = e0.elapsed_time(e1)
+        # keep the GPU loaded for at least ~1.5 s so the clock samples cover a busy GPU
+        t_end = time.time() + max(0.0, 1.5 - elapsed_ms / 1e3)
+        i = args.steps
+        while time.time() < t_end:
+            one(i)
+            i += 1
+            if i % 64 == 0:
+                torch.cuda.synchronize(dev)
+        torch.cuda.synchronize(dev)
+        clocks.stop()
+        code = abi.check_status(stream)
+        if code != abi.MLA_OK:
+            raise RuntimeError(f"device status after timing: {abi.status_name(code)}")
+
+        # ---- the attention kernel alone, per launch, on its own stream
+        attn_ms = []
+        for i in range(args.steps):
+            d, st = dws[i % replicas], steps[i % replicas]
+            abi.absorb_q(d.dims, d.q_nope, d.q_pe, d.kv_len, d.w_uk, st.q_abs, stream)
+            a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a0.record(stream)
+            abi.decode_attn(d.dims, d.cache, d.kv_len, d.max_kv_len, st.q_abs, st.o_part, st.lse_part, S, stream)
+            a1.record(stream)
+            attn_ms.append((a0, a1))
+        torch.cuda.synchronize(dev)
+        attn_ms = [a.elapsed_time(b) for a, b in attn_ms]
+
+        # ---- end to end through the public API with host buffers
+        host_in = {k: getattr(w, k).pin_memory() for k in ("q_nope", "q_pe", "c_new", "kr_new", "kv_len", "start_pos")}
+        out_dev = steps[0].out if steps[0].out is not None else steps[0].o
+        host_out = torch.empty(out_dev.shape, dtype=out_dev.dtype).pin_memory()
+        h2d = sum(t.numel() * t.element_size() for t in host_in.values())
+        d2h = host_out.numel() * host_out.element_size()
+
+        def e2e_step(i):
+            d, st = dws[i % replicas], steps[i % replicas]
+            for k, t in host_in.items():
+                getattr(d, k).copy_(t, non_blocking=True)
+            res = st(d.q_nope, d.q_pe, d.kv_len, d.w_uk, d.w_uv, d.w_o, c_new=d.c_new, kr_new=d.kr_new,
+                     start_pos=d.start_pos)
+            host_out.copy_(res, non_blocking=True)
+
+        for i in range(3):
+            e2e_step(i)
+        torch.cuda.synchronize(dev)
+        barrier(world)
+        x0, x1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        x0.record(stream)
+        for i in range(args.steps):
+            e2e_step(i)
+        x1.record(stream)
+        torch.cuda.synchronize(dev)
+        e2e_ms = x0.elapsed_time(x1)
+        assert abi.check_status(stream) == abi.MLA_OK
+
+    max_ms = max_over_ranks(elapsed_ms, world, dev)
+    max_e2e = max_over_ranks(e2e_ms, world, dev)
+    total_bytes = sum_over_ranks(float(cache_bytes) * args.steps, world, dev)
+    ms_step = max_ms / args.steps
+    attn_avg_ms = sum(attn_ms) / len(attn_ms)
+    peaks = load_peaks()
+    achieved = cache_bytes / (attn_avg_ms * 1e-3) / 1e9
+    launches_per_step = 1 + 2 + 1 + 1 + (2 if shape.hidden else 1)
+    line = {
+        "metric": METRIC,
+        "value": round(total_bytes / (max_ms * 1e-3) / 1e9, 2),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_step, 6),
+        "us_per_step": round(ms_step * 1e3, 3),
+        "attn_us_per_launch": round(attn_avg_ms * 1e3, 3),
+        "queries_per_s": round(world * shape.batch * shape.q_len / (ms_step * 1e-3), 1),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) caches and queries, N(0,1/sqrt(fan_in)) weights)",
+        "config": {
+            "workload": shape.name, "batch": shape.batch, "q_len": shape.q_len, "heads": shape.num_heads,
+            "kv_groups": shape.num_kv_groups, "rank": shape.rank, "d_rope": shape.d_rope, "d_nope": shape.d_nope,
+            "d_v": shape.d_v, "hidden": shape.hidden,
+            "kv_len": (shape.kv_lo if shape.kv_lo == shape.kv_hi else [shape.kv_lo, shape.kv_hi]),
+            "layout": "paged(64)" if shape.paged else "contiguous", "num_splits": S,
+            "cache_bytes_per_step": cache_bytes,
+            "l2": f"inputs rotate over {replicas} replicas of {per_replica / 2**20:.1f} MiB (> 2x L2 of "
+                  f"{l2 / 2**20:.0f} MiB); no flush",
+            "cuda_graph": graphs is not None, "parallelism": f"replicas{world}",
+        },
+        "roofline": {
+            "bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+            "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": None,
+            "peak_source": peaks["source"], "kernel": "mla_decode_attn",
+            "bytes_per_launch": cache_bytes,
+        },
+        "clocks": clocks.summary(),
+        "e2e": {"value": round(total_bytes / (max_e2e * 1e-3) / 1e9, 2), "unit": "GB/s",
+                "us_per_step": round(max_e2e / args.steps * 1e3, 3),
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": launches_per_step * args.steps,
+    }
+    return line, w
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": p["hbm_gbs"], "bf16_tflops": p["bf16_tflops"], "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "source": "fallback"}
+
+
+# ---------------------------------------------------------------- the oracle on the host
+
+def oracle_sample(w, budget_s: float = 20.0):
+    """Run the fp64 oracle on growing subsets of the workload's sequences until
+    about `budget_s` seconds of CPU work have been measured.  Returns
+    (GB/s of cache processed, threads, description)."""
+    import numpy as np
+    from oracle import oracle as orc
+    from tests.helpers import bits, dims_of, oracle_cache
+
+    dims = dims_of(w)
+    cache = oracle_cache(w)
+    orc.cache_append(dims, cache, bits(w.c_new), bits(w.kr_new), w.start_pos.numpy())
+    args = (bits(w.q_nope), bits(w.q_pe), w.kv_len.numpy(), bits(w.w_uk), bits(w.w_uv),
+            None if w.w_o is None else bits(w.w_o))
+    order = list(np.argsort(-w.kv_len.numpy()))  # longest first, spread over the length mix
+    order = order[::2] + order[1::2]
+    done, spent, nbytes = 0, 0.0, 0
+    per_tok = (w.shape.rank + w.shape.d_rope) * 2
+    while done < len(order) and spent < budget_s:
+        take = max(1, min(len(order) - done, 2 ** max(0, int(math.log2(done + 1)))))
+        seqs = order[done:done + take]
+        t0 = time.perf_counter()
+        orc.mla_decode(dims, cache, *args[:5], args[5], seqs=seqs)
+        spent += time.perf_counter() - t0
+        nbytes += int(w.kv_len.numpy()[seqs].sum()) * per_tok
+        done += take
+    desc = (f"{done} of {len(order)} sequences of {w.shape.name} ({nbytes / 1e6:.1f} MB of cache), "
+            f"fp64 non-absorbed oracle incl. W_O")
+    return nbytes / spent / 1e9, orc.num_threads(), desc, spent
+
+
+def run_reference(args, rank, world):
+    """The reference arm: the CPU oracle, timed as it stands on the host cores."""
+    from paper_2607_27269_gb300 import workloads as wl
+    from oracle import oracle as orc
+    from tests.helpers import bits, dims_of, oracle_cache
+
+    if rank != 0:
+        return None
+    shape = wl.SHAPES[args.workload]
+    w = wl.make(shape, seed=args.seed)
+    dims = dims_of(w)
+    cache = oracle_cache(w)
+    orc.cache_append(dims, cache, bits(w.c_new), bits(w.kr_new), w.start_pos.numpy())
+    inputs = (bits(w.q_nope), bits(w.q_pe), w.kv_len.numpy(), bits(w.w_uk), bits(w.w_uv),
+              None if w.w_o is None else bits(w.w_o))
+    # one step = the oracle on a bounded sample of the workload's sequences,
+    # sized from one probe so that warm-up + steps stay within about 2 minutes
+    import numpy as np
+    order = list(np.argsort(-w.kv_len.numpy()))
+    t0 = time.perf_counter()
+    orc.mla_decode(dims, cache, *inputs[:5], inputs[5], seqs=order[:1])
+    one = max(time.perf_counter() - t0, 1e-4)
+    budget = 120.0 / max(args.steps + args.warmup, 1)
+    n = int(max(1, min(len(order), budget / one)))
+    seqs = order[:n]
+    per_tok = (shape.rank + shape.d_rope) * 2
+    nbytes = int(w.kv_len.numpy()[seqs].sum()) * per_tok
+    for _ in range(args.warmup):
+        orc.mla_decode(dims, cache, *inputs[:5], inputs[5], seqs=seqs)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        orc.mla_decode(dims, cache, *inputs[:5], inputs[5], seqs=seqs)
+    el = time.perf_counter() - t0
+    value = nbytes * args.steps / el / 1e9
+    sample = f"{n} of {len(order)} sequences of {shape.name} per step, fp64 non-absorbed oracle incl. W_O"
+    return {
+        "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(el / args.steps * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": shape.name, "sample": sample},
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": orc.num_threads(), "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        if args.impl == "reference":
+            if rank != 0:
+                return 0
+            world = 1
+        else:
+            import torch
+            torch.cuda.set_device(local)
+            dist.init_process_group("nccl")
+    if args.impl == "reference":
+        line = run_reference(args, rank, world)
+        if line is not None:
+            print(json.dumps(line), flush=True)
+        return 0
+    line, w = run_ours(args, rank, world, local)
+    if rank == 0:
+        if world == 1 and not args.no_cpu_baseline:
+            v, cores, desc, spent = oracle_sample(w)
+            line["cpu_baseline"] = {"value": round(v, 4), "unit": "GB/s", "cores": cores, "kind": "oracle",
+                                    "sample": desc, "seconds": round(spent, 2)}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,268 @@
+"""ctypes binding of libgbmla.so (``include/gbmla.h``).
+
+Argument marshalling only: every function here forwards torch tensors' device
+pointers, sizes and the current CUDA stream to the C entry point of the same
+name and raises ``MlaError`` on a non-OK status.  All compute happens in the
+library's kernels.  PyTorch supplies device memory and streams.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from dataclasses import dataclass
+from typing import Optional
+
+import torch
+
+from . import build as _build
+
+MLA_OK, MLA_ERR_INVALID_ARG, MLA_ERR_UNSUPPORTED, MLA_ERR_CUDA, MLA_ERR_DEVICE_BOUNDS, MLA_ERR_DEVICE_TIMEOUT = range(6)
+SPLIT_TILE = 128
+EXPORTS = ("mla_workspace_size", "mla_cache_append", "mla_absorb_q", "mla_decode_attn", "mla_combine",
+           "mla_out_proj", "mla_check_status", "mla_selftest_wait_timeout", "mla_status_str")
+
+
+class MlaError(RuntimeError):
+    def __init__(self, where: str, code: int, name: str):
+        super().__init__(f"{where}: {name}")
+        self.code = code
+        self.name = name
+
+
+class MlaDims(ctypes.Structure):
+    _fields_ = [("num_heads", ctypes.c_int32), ("num_kv_groups", ctypes.c_int32), ("d_nope", ctypes.c_int32),
+                ("d_rope", ctypes.c_int32), ("d_v", ctypes.c_int32), ("rank", ctypes.c_int32),
+                ("hidden", ctypes.c_int32), ("sm_scale", ctypes.c_float), ("rope_style", ctypes.c_int32),
+                ("rope_base", ctypes.c_float)]
+
+
+class MlaCache(ctypes.Structure):
+    _fields_ = [("c_kv", ctypes.c_void_p), ("k_rope", ctypes.c_void_p), ("c_tok_stride", ctypes.c_int64),
+                ("r_tok_stride", ctypes.c_int64), ("c_blk_stride", ctypes.c_int64), ("r_blk_stride", ctypes.c_int64),
+                ("block_table", ctypes.c_void_p), ("bt_stride", ctypes.c_int32), ("page_size", ctypes.c_int32),
+                ("num_pages", ctypes.c_int32), ("capacity", ctypes.c_int32)]
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def lib(auto_build: bool = True):
+    """The loaded library (built first if missing or stale and ``auto_build``)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            path = _build.build() if auto_build else _build.LIB
+            if not os.path.exists(path):
+                raise RuntimeError(f"libgbmla.so is missing at {path}; run paper_2607_27269_gb300.build.build()")
+            L = ctypes.CDLL(path)
+            vp, i32, i64, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
+            P = ctypes.POINTER
+            L.mla_status_str.restype = ctypes.c_char_p
+            L.mla_status_str.argtypes = [ctypes.c_int]
+            L.mla_workspace_size.argtypes = [P(MlaDims), i32, i32, i32, i32, P(sz), P(sz), P(i32)]
+            L.mla_cache_append.argtypes = [P(MlaDims), P(MlaCache), i32, i32, vp, vp, vp, vp]
+            L.mla_absorb_q.argtypes = [P(MlaDims), i32, i32, vp, vp, vp, vp, vp, vp]
+            L.mla_decode_attn.argtypes = [P(MlaDims), P(MlaCache), i32, i32, vp, i32, vp, i32, vp, vp, vp]
+            L.mla_combine.argtypes = [P(MlaDims), i32, i32, i32, vp, i32, vp, vp, vp, vp, vp]
+            L.mla_out_proj.argtypes = [P(MlaDims), i32, i32, vp, vp, vp, vp, vp, vp]
+            L.mla_check_status.argtypes = [vp]
+            L.mla_selftest_wait_timeout.argtypes = [i64, vp]
+            for name in EXPORTS[:-1]:
+                getattr(L, name).restype = ctypes.c_int
+            _lib = L
+        return _lib
+
+
+def status_name(code: int) -> str:
+    return lib().mla_status_str(code).decode()
+
+
+def _check(where: str, code: int):
+    if code != MLA_OK:
+        raise MlaError(where, code, status_name(code))
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _p(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("tensor must live on the GPU")
+    if not t.is_contiguous():
+        raise ValueError("tensor must be contiguous")
+    return t.data_ptr()
+
+
+@dataclass
+class Dims:
+    num_heads: int
+    num_kv_groups: int
+    d_nope: int
+    d_rope: int
+    d_v: int
+    rank: int
+    hidden: int = 0
+    sm_scale: float = 1.0
+    rope_style: int = 0
+    rope_base: float = 10000.0
+
+    def c(self) -> MlaDims:
+        return MlaDims(self.num_heads, self.num_kv_groups, self.d_nope, self.d_rope, self.d_v, self.rank,
+                       self.hidden, self.sm_scale, self.rope_style, self.rope_base)
+
+
+@dataclass
+class Cache:
+    """Device cache: ``c_kv`` [blocks, block_tokens, r] and ``k_rope``
+    [blocks, block_tokens, d_rope] bf16 (or strided views of one fused
+    buffer), blocks = sequences (contiguous) or pages (paged)."""
+    c_kv: torch.Tensor
+    k_rope: torch.Tensor
+    capacity: int
+    block_table: Optional[torch.Tensor] = None
+    page_size: int = 0
+    num_pages: int = 0
+
+    def c(self) -> MlaCache:
+        c, k = self.c_kv, self.k_rope
+        for t in (c, k):
+            if not t.is_cuda or t.dtype != torch.bfloat16 or t.dim() != 3 or t.stride(2) != 1:
+                raise ValueError("cache tensors must be 3-d bf16 CUDA tensors with unit inner stride")
+        bt = self.block_table
+        return MlaCache(c.data_ptr(), k.data_ptr(), c.stride(1), k.stride(1), c.stride(0), k.stride(0),
+                        _p(bt), 0 if bt is None else bt.shape[1], self.page_size, self.num_pages, self.capacity)
+
+
+def workspace_size(dims: Dims, batch: int, q_len: int, max_kv_len: int, num_splits: int = 0):
+    """(o_part_bytes, lse_part_bytes, num_splits_used)."""
+    ob, lb, s = ctypes.c_size_t(), ctypes.c_size_t(), ctypes.c_int32()
+    _check("mla_workspace_size", lib().mla_workspace_size(ctypes.byref(dims.c()), batch, q_len, max_kv_len,
+                                                          num_splits, ctypes.byref(ob), ctypes.byref(lb),
+                                                          ctypes.byref(s)))
+    return ob.value, lb.value, s.value
+
+
+def cache_append(dims: Dims, cache: Cache, c_new: torch.Tensor, kr_new: torch.Tensor, start_pos: torch.Tensor,
+                 stream=None):
+    batch, n_new = c_new.shape[0], c_new.shape[1]
+    _check("mla_cache_append", lib().mla_cache_append(ctypes.byref(dims.c()), ctypes.byref(cache.c()), batch, n_new,
+                                                      _p(c_new), _p(kr_new), _p(start_pos), _stream(stream)))
+
+
+def absorb_q(dims: Dims, q_nope: torch.Tensor, q_pe: torch.Tensor, kv_len: torch.Tensor, w_uk: torch.Tensor,
+             q_abs: torch.Tensor, stream=None):
+    batch, q_len = q_nope.shape[0], q_nope.shape[1]
+    _check("mla_absorb_q", lib().mla_absorb_q(ctypes.byref(dims.c()), batch, q_len, _p(q_nope), _p(q_pe),
+                                              _p(kv_len), _p(w_uk), _p(q_abs), _stream(stream)))
+
+
+def decode_attn(dims: Dims, cache: Cache, kv_len: torch.Tensor, max_kv_len: int, q_abs: torch.Tensor,
+                o_part: torch.Tensor, lse_part: torch.Tensor, num_splits: int = 0, stream=None):
+    batch, q_len = q_abs.shape[0], q_abs.shape[1]
+    _check("mla_decode_attn", lib().mla_decode_attn(ctypes.byref(dims.c()), ctypes.byref(cache.c()), batch, q_len,
+                                                    _p(kv_len), max_kv_len, _p(q_abs), num_splits, _p(o_part),
+                                                    _p(lse_part), _stream(stream)))
+
+
+def combine(dims: Dims, batch: int, q_len: int, kv_len: torch.Tensor, max_kv_len: int, o_part: torch.Tensor,
+            lse_part: torch.Tensor, o_lat: torch.Tensor, lse: Optional[torch.Tensor] = None, num_splits: int = 0,
+            stream=None):
+    _check("mla_combine", lib().mla_combine(ctypes.byref(dims.c()), batch, q_len, num_splits, _p(kv_len), max_kv_len,
+                                            _p(o_part), _p(lse_part), _p(o_lat), _p(lse), _stream(stream)))
+
+
+def out_proj(dims: Dims, o_lat: torch.Tensor, w_uv: torch.Tensor, w_o: Optional[torch.Tensor], o: torch.Tensor,
+             out: Optional[torch.Tensor], stream=None):
+    batch, q_len = o_lat.shape[0], o_lat.shape[1]
+    _check("mla_out_proj", lib().mla_out_proj(ctypes.byref(dims.c()), batch, q_len, _p(o_lat), _p(w_uv), _p(w_o),
+                                              _p(o), _p(out), _stream(stream)))
+
+
+def check_status(stream=None) -> int:
+    """Synchronise the stream and return (and clear) the device status code."""
+    return lib().mla_check_status(_stream(stream))
+
+
+def selftest_wait_timeout(limit_ns: int, stream=None):
+    _check("mla_selftest_wait_timeout", lib().mla_selftest_wait_timeout(int(limit_ns), _stream(stream)))
+
+
+class DecodeStep:
+    """One decode step of an MLA layer through the five entry points, with
+    every intermediate buffer allocated once (by PyTorch) up front:
+    append -> absorb -> split-KV attention -> combine -> up/out projection."""
+
+    def __init__(self, dims: Dims, cache: Cache, batch: int, q_len: int, max_kv_len: int, num_splits: int = 0,
+                 device=None):
+        self.dims, self.cache = dims, cache
+        self.batch, self.q_len, self.max_kv_len = batch, q_len, max_kv_len
+        dev = device or cache.c_kv.device
+        ob, lb, s = workspace_size(dims, batch, q_len, max_kv_len, num_splits)
+        self.num_splits = s
+        H, r, dr = dims.num_heads, dims.rank, dims.d_rope
+        slots = max(ob // 4 // max(q_len * H * r, 1), 1)
+        self.q_abs = torch.empty(batch, q_len, H, r + dr, dtype=torch.bfloat16, device=dev)
+        self.o_part = torch.empty(slots, q_len, H, r, dtype=torch.float32, device=dev)
+        self.lse_part = torch.empty(slots, q_len, H, dtype=torch.float32, device=dev)
+        self.o_lat = torch.empty(batch, q_len, H, r, dtype=torch.float32, device=dev)
+        self.lse = torch.empty(batch, q_len, H, dtype=torch.float32, device=dev)
+        self.o = torch.empty(batch, q_len, H, dims.d_v, dtype=torch.bfloat16, device=dev)
+        self.out = (torch.empty(batch, q_len, dims.hidden, dtype=torch.bfloat16, device=dev)
+                    if dims.hidden else None)
+
+    def __call__(self, q_nope, q_pe, kv_len, w_uk, w_uv, w_o=None, c_new=None, kr_new=None, start_pos=None,
+                 stream=None):
+        d = self.dims
+        if c_new is not None:
+            cache_append(d, self.cache, c_new, kr_new, start_pos, stream)
+        absorb_q(d, q_nope, q_pe, kv_len, w_uk, self.q_abs, stream)
+        decode_attn(d, self.cache, kv_len, self.max_kv_len, self.q_abs, self.o_part, self.lse_part, self.num_splits,
+                    stream)
+        combine(d, self.batch, self.q_len, kv_len, self.max_kv_len, self.o_part, self.lse_part, self.o_lat, self.lse,
+                self.num_splits, stream)
+        out_proj(d, self.o_lat, w_uv, w_o if d.hidden else None, self.o, self.out if d.hidden else None, stream)
+        return self.out if (d.hidden and w_o is not None) else self.o
+
+
+@dataclass
+class DeviceWorkload:
+    """A workload's tensors on the GPU plus its Dims and Cache descriptors."""
+    dims: Dims
+    cache: Cache
+    batch: int
+    q_len: int
+    max_kv_len: int
+    kv_len: torch.Tensor
+    start_pos: torch.Tensor
+    w_uk: torch.Tensor
+    w_uv: torch.Tensor
+    w_o: Optional[torch.Tensor]
+    q_nope: torch.Tensor
+    q_pe: torch.Tensor
+    c_new: torch.Tensor
+    kr_new: torch.Tensor
+
+
+def to_device(w, device="cuda") -> DeviceWorkload:
+    """Copy a ``workloads.Workload`` to the GPU (plain host-to-device copies)."""
+    s = w.shape
+    dims = Dims(s.num_heads, s.num_kv_groups, s.d_nope, s.d_rope, s.d_v, s.rank, s.hidden, s.sm_scale,
+                s.rope_style, s.rope_base)
+    put = lambda t: None if t is None else t.to(device)
+    bt = put(w.block_table)
+    cache = Cache(put(w.c_kv), put(w.k_rope), w.capacity, bt, s.page_size if s.paged else 0, w.num_pages)
+    batch, q_len = w.kv_len.numel(), w.q_nope.shape[1]
+    return DeviceWorkload(dims, cache, batch, q_len, int(w.kv_len.max()) if batch else q_len, put(w.kv_len),
+                          put(w.start_pos), put(w.w_uk), put(w.w_uv), put(w.w_o), put(w.q_nope), put(w.q_pe),
+                          put(w.c_new), put(w.kr_new))

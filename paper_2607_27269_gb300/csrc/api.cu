@@ -1,0 +1,283 @@
+// The C ABI of libgbmla.so (include/gbmla.h): host-side argument checks,
+// split resolution, the per-device status word and the launches.
+#include <math.h>
+#include <mutex>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace gbmla {
+namespace {
+
+// Sticky status word, one per device (a __device__ variable lives once per
+// device context).  Kernels receive its device address.
+__device__ unsigned g_status_word;
+
+constexpr int kMaxDevices = 64;
+std::mutex g_mutex;
+unsigned *g_status_ptr[kMaxDevices];
+int g_sm_count[kMaxDevices];
+
+// Device address of this device's status word and its SM count, looked up
+// once per device with that device current.
+mla_status device_info(unsigned **status, int *sms)
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return MLA_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(g_mutex);
+    if (!g_status_ptr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return MLA_ERR_CUDA;
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return MLA_ERR_CUDA;
+        g_status_ptr[dev] = static_cast<unsigned *>(p);
+        g_sm_count[dev] = n;
+    }
+    if (status) *status = g_status_ptr[dev];
+    if (sms) *sms = g_sm_count[dev];
+    return MLA_OK;
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+mla_status check_dims(const mla_dims *d)
+{
+    if (!d) return MLA_ERR_INVALID_ARG;
+    if (d->num_heads <= 0 || d->num_kv_groups <= 0 || d->num_heads % d->num_kv_groups) return MLA_ERR_INVALID_ARG;
+    if (d->d_nope <= 0 || d->d_v <= 0 || d->rank <= 0 || d->d_rope < 0 || d->hidden < 0) return MLA_ERR_INVALID_ARG;
+    if (!(d->sm_scale > 0.f) || !isfinite(d->sm_scale)) return MLA_ERR_INVALID_ARG;
+    if (!(d->rope_base > 1.f) || !isfinite(d->rope_base)) return MLA_ERR_INVALID_ARG;
+    if (d->rope_style != 0 && d->rope_style != 1) return MLA_ERR_INVALID_ARG;
+    if (d->d_rope != 32 && d->d_rope != 64) return MLA_ERR_UNSUPPORTED;
+    if (d->rank % 64 || d->rank > 512) return MLA_ERR_UNSUPPORTED;
+    if (d->d_nope % 8 || d->d_nope > 256 || d->d_v % 8 || d->d_v > 256) return MLA_ERR_UNSUPPORTED;
+    if (d->num_heads > 128) return MLA_ERR_UNSUPPORTED;
+    return MLA_OK;
+}
+
+mla_status check_cache(const mla_dims *d, const mla_cache *c, CacheView *v)
+{
+    if (!c || !c->c_kv || !c->k_rope) return MLA_ERR_INVALID_ARG;
+    if (!aligned16(c->c_kv) || !aligned16(c->k_rope)) return MLA_ERR_INVALID_ARG;
+    if (c->c_tok_stride % 8 || c->r_tok_stride % 8 || c->c_blk_stride % 8 || c->r_blk_stride % 8)
+        return MLA_ERR_INVALID_ARG;
+    if (c->c_tok_stride < d->rank || c->r_tok_stride < d->d_rope || c->c_blk_stride < 0 || c->r_blk_stride < 0)
+        return MLA_ERR_INVALID_ARG;
+    if (c->capacity <= 0) return MLA_ERR_INVALID_ARG;
+    if (c->block_table) {
+        if (c->page_size != 64) return MLA_ERR_UNSUPPORTED;
+        if (c->num_pages <= 0 || c->bt_stride <= 0) return MLA_ERR_INVALID_ARG;
+        if (static_cast<int64_t>(c->bt_stride) * c->page_size < c->capacity) return MLA_ERR_INVALID_ARG;
+    }
+    v->c_kv = c->c_kv;
+    v->k_rope = c->k_rope;
+    v->c_tok = c->c_tok_stride;
+    v->r_tok = c->r_tok_stride;
+    v->c_blk = c->c_blk_stride;
+    v->r_blk = c->r_blk_stride;
+    v->block_table = c->block_table;
+    v->bt_stride = c->bt_stride;
+    v->page_size = c->page_size;
+    v->num_pages = c->num_pages;
+    v->capacity = c->capacity;
+    return MLA_OK;
+}
+
+// Partitions used for (dims, batch, q_len, max_kv_len): `requested` if > 0,
+// otherwise about two blocks per SM across the query groups, never more
+// partitions than tiles.
+int resolve_splits(const mla_dims *d, int batch, int q_len, int max_kv_len, int requested, int sms)
+{
+    const int64_t max_tiles = static_cast<int64_t>(batch) * ((max_kv_len + MLA_SPLIT_TILE - 1) / MLA_SPLIT_TILE);
+    if (requested > 0) return requested;
+    const int rows = q_len * d->num_heads;
+    const int groups = (rows + kSimtRows - 1) / kSimtRows;
+    int64_t s = (2 * static_cast<int64_t>(sms) + groups - 1) / groups;
+    if (s > max_tiles) s = max_tiles;
+    if (s < 1) s = 1;
+    return static_cast<int>(s);
+}
+
+mla_status from_cuda(cudaError_t e) { return e == cudaSuccess ? MLA_OK : MLA_ERR_CUDA; }
+
+__global__ void selftest_wait_kernel(uint64_t limit_ns, unsigned *status)
+{
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x == 0) mbar_init(&bar, 1);
+    __syncthreads();
+    // Nothing arrives on `bar`: the bounded wait must give up.
+    if (!mbar_wait(smem_u32(&bar), 0, limit_ns)) {
+        if (threadIdx.x == 0) record_status(status, kStatusTimeout);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_selftest_wait(int64_t limit_ns, unsigned *status, cudaStream_t st)
+{
+    selftest_wait_kernel<<<1, 32, 0, st>>>(static_cast<uint64_t>(limit_ns), status);
+    return cudaGetLastError();
+}
+
+}  // namespace gbmla
+
+using namespace gbmla;
+
+extern "C" {
+
+const char *mla_status_str(mla_status s)
+{
+    switch (s) {
+    case MLA_OK: return "MLA_OK";
+    case MLA_ERR_INVALID_ARG: return "MLA_ERR_INVALID_ARG";
+    case MLA_ERR_UNSUPPORTED: return "MLA_ERR_UNSUPPORTED";
+    case MLA_ERR_CUDA: return "MLA_ERR_CUDA";
+    case MLA_ERR_DEVICE_BOUNDS: return "MLA_ERR_DEVICE_BOUNDS";
+    case MLA_ERR_DEVICE_TIMEOUT: return "MLA_ERR_DEVICE_TIMEOUT";
+    }
+    return "MLA_ERR_UNKNOWN";
+}
+
+mla_status mla_workspace_size(const mla_dims *dims, int32_t batch, int32_t q_len, int32_t max_kv_len,
+                              int32_t num_splits, size_t *o_part_bytes, size_t *lse_part_bytes,
+                              int32_t *num_splits_used)
+{
+    mla_status s = check_dims(dims);
+    if (s != MLA_OK) return s;
+    if (batch < 0 || q_len < 1 || q_len > 16 || max_kv_len < q_len || num_splits < 0) return MLA_ERR_INVALID_ARG;
+    int sms = 0;
+    if ((s = device_info(nullptr, &sms)) != MLA_OK) return s;
+    const int S = resolve_splits(dims, batch, q_len, max_kv_len, num_splits, sms);
+    const size_t slots = batch > 0 ? static_cast<size_t>(batch) + S - 1 : 0;
+    const size_t rows = static_cast<size_t>(q_len) * dims->num_heads;
+    if (o_part_bytes) *o_part_bytes = slots * rows * dims->rank * sizeof(float);
+    if (lse_part_bytes) *lse_part_bytes = slots * rows * sizeof(float);
+    if (num_splits_used) *num_splits_used = S;
+    return MLA_OK;
+}
+
+mla_status mla_cache_append(const mla_dims *dims, const mla_cache *cache, int32_t batch, int32_t n_new,
+                            const void *c_new, const void *kr_new, const int32_t *start_pos, void *stream)
+{
+    mla_status s = check_dims(dims);
+    if (s != MLA_OK) return s;
+    CacheView v;
+    if ((s = check_cache(dims, cache, &v)) != MLA_OK) return s;
+    if (batch < 0 || n_new < 0 || batch > 65535 || n_new > 65535) return MLA_ERR_INVALID_ARG;
+    if (batch == 0 || n_new == 0) return MLA_OK;
+    if (!c_new || !kr_new || !start_pos || !aligned16(c_new)) return MLA_ERR_INVALID_ARG;
+    unsigned *status = nullptr;
+    if ((s = device_info(&status, nullptr)) != MLA_OK) return s;
+    return from_cuda(launch_append(*dims, v, batch, n_new, c_new, kr_new, start_pos, status,
+                                   static_cast<cudaStream_t>(stream)));
+}
+
+mla_status mla_absorb_q(const mla_dims *dims, int32_t batch, int32_t q_len, const void *q_nope, const void *q_pe,
+                        const int32_t *kv_len, const void *w_uk, void *q_abs, void *stream)
+{
+    mla_status s = check_dims(dims);
+    if (s != MLA_OK) return s;
+    if (batch < 0 || q_len < 1 || q_len > 16) return MLA_ERR_INVALID_ARG;
+    if (batch == 0) return MLA_OK;
+    if (!q_nope || !q_pe || !kv_len || !w_uk || !q_abs) return MLA_ERR_INVALID_ARG;
+    if (static_cast<int64_t>(batch) * q_len > (1 << 30)) return MLA_ERR_UNSUPPORTED;
+    unsigned *status = nullptr;
+    if ((s = device_info(&status, nullptr)) != MLA_OK) return s;
+    return from_cuda(launch_absorb(*dims, batch, q_len, q_nope, q_pe, kv_len, w_uk, q_abs, status,
+                                   static_cast<cudaStream_t>(stream)));
+}
+
+mla_status mla_decode_attn(const mla_dims *dims, const mla_cache *cache, int32_t batch, int32_t q_len,
+                           const int32_t *kv_len, int32_t max_kv_len, const void *q_abs, int32_t num_splits,
+                           float *o_part, float *lse_part, void *stream)
+{
+    mla_status s = check_dims(dims);
+    if (s != MLA_OK) return s;
+    CacheView v;
+    if ((s = check_cache(dims, cache, &v)) != MLA_OK) return s;
+    if (batch < 0 || q_len < 1 || q_len > 16 || num_splits < 0) return MLA_ERR_INVALID_ARG;
+    if (max_kv_len < q_len || max_kv_len > cache->capacity) return MLA_ERR_INVALID_ARG;
+    if (batch == 0) return MLA_OK;
+    if (!kv_len || !q_abs || !o_part || !lse_part || !aligned16(o_part) || !aligned16(q_abs))
+        return MLA_ERR_INVALID_ARG;
+    unsigned *status = nullptr;
+    int sms = 0;
+    if ((s = device_info(&status, &sms)) != MLA_OK) return s;
+    AttnArgs a;
+    a.batch = batch;
+    a.q_len = q_len;
+    a.num_heads = dims->num_heads;
+    a.rank = dims->rank;
+    a.d_rope = dims->d_rope;
+    a.sm_scale = dims->sm_scale;
+    a.kv_len = kv_len;
+    a.max_kv = max_kv_len;
+    a.q_abs = q_abs;
+    a.num_splits = resolve_splits(dims, batch, q_len, max_kv_len, num_splits, sms);
+    a.o_part = o_part;
+    a.lse_part = lse_part;
+    a.cache = v;
+    a.status = status;
+    return from_cuda(launch_attn_simt(a, static_cast<cudaStream_t>(stream)));
+}
+
+mla_status mla_combine(const mla_dims *dims, int32_t batch, int32_t q_len, int32_t num_splits,
+                       const int32_t *kv_len, int32_t max_kv_len, const float *o_part, const float *lse_part,
+                       float *o_lat, float *lse, void *stream)
+{
+    mla_status s = check_dims(dims);
+    if (s != MLA_OK) return s;
+    if (batch < 0 || q_len < 1 || q_len > 16 || num_splits < 0 || max_kv_len < q_len) return MLA_ERR_INVALID_ARG;
+    if (batch == 0) return MLA_OK;
+    if (!kv_len || !o_part || !lse_part || !o_lat || !aligned16(o_part) || !aligned16(o_lat))
+        return MLA_ERR_INVALID_ARG;
+    int sms = 0;
+    if ((s = device_info(nullptr, &sms)) != MLA_OK) return s;
+    const int S = resolve_splits(dims, batch, q_len, max_kv_len, num_splits, sms);
+    // a length above max_kv_len counts as unusable in both kernels
+    return from_cuda(launch_combine(batch, q_len, dims->num_heads, dims->rank, max_kv_len, S, kv_len, o_part,
+                                    lse_part, o_lat, lse, static_cast<cudaStream_t>(stream)));
+}
+
+mla_status mla_out_proj(const mla_dims *dims, int32_t batch, int32_t q_len, const float *o_lat, const void *w_uv,
+                        const void *w_o, void *o, void *out, void *stream)
+{
+    mla_status s = check_dims(dims);
+    if (s != MLA_OK) return s;
+    if (batch < 0 || q_len < 1 || q_len > 16) return MLA_ERR_INVALID_ARG;
+    if (batch == 0) return MLA_OK;
+    if (!o_lat || !w_uv || !o) return MLA_ERR_INVALID_ARG;
+    if (w_o && dims->hidden > 0 && !out) return MLA_ERR_INVALID_ARG;
+    if ((s = device_info(nullptr, nullptr)) != MLA_OK) return s;
+    return from_cuda(launch_out_proj(*dims, batch, q_len, o_lat, w_uv, w_o, o, out,
+                                     static_cast<cudaStream_t>(stream)));
+}
+
+mla_status mla_check_status(void *stream)
+{
+    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return MLA_ERR_CUDA;
+    unsigned *status = nullptr;
+    mla_status s = device_info(&status, nullptr);
+    if (s != MLA_OK) return s;
+    unsigned word = 0;
+    if (cudaMemcpy(&word, status, sizeof word, cudaMemcpyDeviceToHost) != cudaSuccess) return MLA_ERR_CUDA;
+    if (word) {
+        const unsigned zero = 0;
+        if (cudaMemcpy(status, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess) return MLA_ERR_CUDA;
+    }
+    if (word & kStatusTimeout) return MLA_ERR_DEVICE_TIMEOUT;
+    if (word & kStatusBounds) return MLA_ERR_DEVICE_BOUNDS;
+    return MLA_OK;
+}
+
+mla_status mla_selftest_wait_timeout(int64_t limit_ns, void *stream)
+{
+    if (limit_ns < 1000) limit_ns = 1000;
+    if (limit_ns > 1000000000) limit_ns = 1000000000;
+    unsigned *status = nullptr;
+    mla_status s = device_info(&status, nullptr);
+    if (s != MLA_OK) return s;
+    return from_cuda(launch_selftest_wait(limit_ns, status, static_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

@@ -1,0 +1,132 @@
+// Device-side helpers shared by the kernels of libgbmla.so.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/gbmla.h"
+
+namespace gbmla {
+
+// Bits of the sticky per-device status word (read by mla_check_status).
+enum : unsigned { kStatusBounds = 1u, kStatusTimeout = 2u };
+
+// Default limit of every bounded device-side wait (about a second).
+constexpr uint64_t kWaitLimitNs = 1000000000ull;
+
+__device__ __forceinline__ void record_status(unsigned *status, unsigned bits)
+{
+    atomicOr(status, bits);
+}
+
+__device__ __forceinline__ uint64_t global_ns()
+{
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ float bf16_bits_to_float(uint16_t b)
+{
+    return __uint_as_float(static_cast<uint32_t>(b) << 16);
+}
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p)
+{
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// ---------------------------------------------------------------- mbarriers
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar, unsigned count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Wait until the phase with the given parity of the mbarrier at shared
+// address `bar` has completed, for at most `limit_ns` nanoseconds.  Returns
+// false if the limit ran out (the caller records a timeout and winds down).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint64_t limit_ns)
+{
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_ns();
+    for (;;) {
+        for (int i = 0; i < 32; ++i)
+            if (mbar_try_wait(bar, parity)) return true;
+        if (global_ns() - t0 > limit_ns) return false;
+    }
+}
+
+// ---------------------------------------------------------------- split-KV partition
+// Tiles of MLA_SPLIT_TILE tokens of all sequences, in batch order, form one
+// list of T tiles; partition k owns tiles [floor(k*T/S), floor((k+1)*T/S)).
+
+__device__ __forceinline__ int64_t part_begin(int64_t k, int64_t T, int S)
+{
+    return (k * T) / S;
+}
+
+// Largest k whose range starts at or before tile t (the non-empty partition
+// holding tile t).
+__device__ __forceinline__ int part_of_tile(int64_t t, int64_t T, int S)
+{
+    return static_cast<int>(((t + 1) * S - 1) / T);
+}
+
+// Tiles of a sequence with kv cached tokens; a length the kernels cannot
+// serve (kv < q_len or kv > capacity) counts as zero tiles everywhere, so
+// every kernel derives the same partition from the same kv_len.
+__device__ __forceinline__ int64_t seq_tiles(int kv, int q_len, int capacity)
+{
+    if (kv < q_len || kv > capacity || kv <= 0) return 0;
+    return (kv + MLA_SPLIT_TILE - 1) / MLA_SPLIT_TILE;
+}
+
+// Block-wide sum of seq_tiles over sequences [0, n); every thread gets it.
+// Uses `red` (>= 32 int64) of shared scratch.  All threads must call it.
+__device__ __forceinline__ int64_t block_tile_sum(const int32_t *kv_len, int n, int q_len, int capacity,
+                                                  int64_t *red)
+{
+    int64_t acc = 0;
+    for (int b = threadIdx.x; b < n; b += blockDim.x) acc += seq_tiles(kv_len[b], q_len, capacity);
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    __syncthreads();
+    if (lane == 0) red[warp] = acc;
+    __syncthreads();
+    int64_t tot = 0;
+    const int nw = (blockDim.x + 31) >> 5;
+    for (int w = 0; w < nw; ++w) tot += red[w];
+    __syncthreads();
+    return tot;
+}
+
+// RoPE angle pos * theta_k reduced to [-pi, pi] in fp64 before the fp32
+// sincos, so that positions up to 2^31 keep fp32 accuracy.
+__device__ __forceinline__ void rope_cos_sin(int64_t pos, double theta, float *c, float *s)
+{
+    const double two_pi = 6.283185307179586476925286766559;
+    double ang = static_cast<double>(pos) * theta;
+    ang -= two_pi * rint(ang / two_pi);
+    sincosf(static_cast<float>(ang), s, c);
+}
+
+// theta_k = base^(-2k/d) in fp64.
+__device__ __forceinline__ double rope_theta(int k, int d, float base)
+{
+    return exp2(-(2.0 * k / d) * log2(static_cast<double>(base)));
+}
+
+}  // namespace gbmla

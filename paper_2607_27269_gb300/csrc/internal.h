@@ -1,0 +1,53 @@
+// Host-side declarations shared by the C-ABI glue (api.cu) and the kernel
+// translation units.  Not part of the public ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/gbmla.h"
+
+namespace gbmla {
+
+// Cache description as the kernels take it (validated by api.cu).
+struct CacheView {
+    const void *c_kv;
+    const void *k_rope;
+    int64_t c_tok, r_tok, c_blk, r_blk;   // strides in elements
+    const int32_t *block_table;           // nullptr: contiguous
+    int32_t bt_stride, page_size, num_pages, capacity;
+};
+
+struct AttnArgs {
+    int32_t batch, q_len, num_heads, rank, d_rope;
+    float sm_scale;
+    const int32_t *kv_len;
+    int32_t max_kv;         // lengths above this (<= capacity) are unusable
+    const void *q_abs;      // bf16 [B, q, H, rank + d_rope]
+    int32_t num_splits;     // S (resolved)
+    float *o_part, *lse_part;
+    CacheView cache;
+    unsigned *status;
+};
+
+cudaError_t launch_append(const mla_dims &d, const CacheView &c, int batch, int n_new, const void *c_new,
+                          const void *kr_new, const int32_t *start_pos, unsigned *status, cudaStream_t st);
+
+cudaError_t launch_absorb(const mla_dims &d, int batch, int q_len, const void *q_nope, const void *q_pe,
+                          const int32_t *kv_len, const void *w_uk, void *q_abs, unsigned *status,
+                          cudaStream_t st);
+
+// CUDA-core attention core; `qgroups` query groups of kSimtRows rows each.
+constexpr int kSimtRows = 16;
+cudaError_t launch_attn_simt(const AttnArgs &a, cudaStream_t st);
+
+cudaError_t launch_combine(int batch, int q_len, int num_heads, int rank, int max_kv, int num_splits,
+                           const int32_t *kv_len, const float *o_part, const float *lse_part, float *o_lat,
+                           float *lse, cudaStream_t st);
+
+cudaError_t launch_out_proj(const mla_dims &d, int batch, int q_len, const float *o_lat, const void *w_uv,
+                            const void *w_o, void *o, void *out, cudaStream_t st);
+
+cudaError_t launch_selftest_wait(int64_t limit_ns, unsigned *status, cudaStream_t st);
+
+}  // namespace gbmla

@@ -1,0 +1,208 @@
+"""GPU parity: every entry point of the C ABI against the fp64 oracle on the
+same seeded inputs.
+
+Bars: cache append and paged addressing bit-exact (latent rows are copies;
+rotated keys within one bf16 rounding of the exact fp64 rotation); every
+floating-point output within max|d| <= 2e-2 max|ref| and mean relative error
+sum|d| / sum|ref| <= 5e-3.
+"""
+from __future__ import annotations
+
+import dataclasses
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as orc
+from paper_2607_27269_gb300 import abi
+from paper_2607_27269_gb300 import workloads as wl
+from tests.helpers import bf16_to_f64, bits, dims_of, oracle_cache, oracle_step, rel_errors
+
+pytestmark = pytest.mark.gpu
+
+MAX_TOL, MEAN_TOL = 2e-2, 5e-3
+
+
+def assert_close(got, ref, what):
+    mx, mean = rel_errors(got, ref)
+    assert mx <= MAX_TOL and mean <= MEAN_TOL, f"{what}: max {mx:.3e} mean {mean:.3e}"
+    return mx, mean
+
+
+def run_step(dw: abi.DeviceWorkload, num_splits=0, append=True):
+    step = abi.DecodeStep(dw.dims, dw.cache, dw.batch, dw.q_len, dw.max_kv_len, num_splits)
+    kw = dict(c_new=dw.c_new, kr_new=dw.kr_new, start_pos=dw.start_pos) if append else {}
+    step(dw.q_nope, dw.q_pe, dw.kv_len, dw.w_uk, dw.w_uv, dw.w_o, **kw)
+    code = abi.check_status()
+    assert code == abi.MLA_OK, abi.status_name(code)
+    return step
+
+
+def test_bounded_wait_times_out_and_reports():
+    abi.check_status()
+    abi.selftest_wait_timeout(2_000_000)                 # 2 ms, nothing ever signals the barrier
+    assert abi.check_status() == abi.MLA_ERR_DEVICE_TIMEOUT
+    assert abi.check_status() == abi.MLA_OK              # the word is cleared by the read
+
+
+@pytest.mark.parametrize("name", wl.ORDER)
+def test_cache_append_bit_exact(name):
+    w = wl.small(name, seed=11)
+    dw = abi.to_device(w)
+    abi.cache_append(dw.dims, dw.cache, dw.c_new, dw.kr_new, dw.start_pos)
+    assert abi.check_status() == abi.MLA_OK
+    cache = oracle_cache(w)
+    orc.cache_append(dims_of(w), cache, bits(w.c_new), bits(w.kr_new), w.start_pos.numpy())
+    got_c, got_r = bits(dw.cache.c_kv.cpu()), bits(dw.cache.k_rope.cpu())
+    # latent rows and every untouched row: identical bits
+    assert np.array_equal(got_c, cache.c_kv)
+    diff = got_r != cache.k_rope
+    # rotated keys: the GPU rotates in fp32, the oracle in fp64; both round once
+    # to bf16, so they may differ by one unit in the last place, nowhere else
+    if diff.any():
+        a = got_r[diff].astype(np.int32)
+        b = cache.k_rope[diff].astype(np.int32)
+        assert np.all(np.abs(a - b) <= 1), "rotated key off by more than one bf16 ulp"
+        assert diff.mean() < 0.01
+    untouched = np.ones(got_r.shape[:2], bool)
+    s = w.shape
+    for bi in range(w.kv_len.numel()):
+        for t in range(int(w.start_pos[bi]), int(w.kv_len[bi])):
+            if s.paged:
+                untouched[int(w.block_table[bi, t // s.page_size]), t % s.page_size] = False
+            else:
+                untouched[bi, t] = False
+    assert not diff[untouched].any()
+
+
+@pytest.mark.parametrize("name", wl.ORDER)
+def test_absorb_q(name):
+    w = wl.small(name, seed=12)
+    dw = abi.to_device(w)
+    s = w.shape
+    q_abs = torch.empty(dw.batch, dw.q_len, s.num_heads, s.rank + s.d_rope, dtype=torch.bfloat16, device="cuda")
+    abi.absorb_q(dw.dims, dw.q_nope, dw.q_pe, dw.kv_len, dw.w_uk, q_abs)
+    assert abi.check_status() == abi.MLA_OK
+    q_lat, q_rot = orc.absorb_q(dims_of(w), bits(w.q_nope), bits(w.q_pe), w.kv_len.numpy(), bits(w.w_uk))
+    got = bf16_to_f64(bits(q_abs.cpu()))
+    assert_close(got[..., :s.rank], q_lat, "q_lat")
+    # the rotated positional query: one fp32 rotation rounded to bf16
+    ref = q_rot
+    ulp = 2.0 ** (np.floor(np.log2(np.maximum(np.abs(ref), 1e-30))) - 7)
+    assert np.all(np.abs(got[..., s.rank:] - ref) <= ulp + 1e-6)
+
+
+@pytest.mark.parametrize("name", wl.ORDER)
+def test_decode_step_matches_oracle(name):
+    w = wl.small(name, seed=13)
+    dw = abi.to_device(w)
+    step = run_step(dw)
+    ref = oracle_step(w)
+    assert_close(step.o_lat.cpu().numpy(), ref["o_lat"], "o_lat")
+    assert_close(step.lse.cpu().numpy(), ref["lse"], "lse")
+    assert_close(bf16_to_f64(bits(step.o.cpu())), ref["o"], "o")
+    if w.w_o is not None:
+        assert_close(bf16_to_f64(bits(step.out.cpu())), ref["out"], "out")
+
+
+@pytest.mark.parametrize("name", ["qwen05b_b16_h14_r256_t2048", "llama1b_paged_b128_h32_r512_t128_8192"])
+def test_split_count_invariance(name):
+    w = wl.small(name, seed=14)
+    outs = []
+    for S in (1, 2, 7, 0):
+        dw = abi.to_device(w)
+        step = run_step(dw, num_splits=S)
+        outs.append((step.o_lat.cpu().numpy().astype(np.float64), step.lse.cpu().numpy().astype(np.float64)))
+    for o, l in outs[1:]:
+        assert rel_errors(o, outs[0][0])[0] < 1e-5
+        assert np.abs(l - outs[0][1]).max() < 1e-5
+
+
+def test_paged_equals_contiguous_bitwise():
+    """The same logical cache, paged through a shuffled block table or laid out
+    contiguously, gives bit-identical attention outputs."""
+    shape = wl.SHAPES["llama1b_paged_b128_h32_r512_t128_8192"]
+    wp = wl.make(shape, seed=15, batch=5, kv_range=(70, 650))
+    s = shape
+    cap = int(wp.kv_len.max())
+    c = torch.zeros(5, cap, s.rank, dtype=torch.bfloat16)
+    r = torch.zeros(5, cap, s.d_rope, dtype=torch.bfloat16)
+    for b in range(5):
+        for t in range(int(wp.kv_len[b])):
+            pg = int(wp.block_table[b, t // s.page_size])
+            c[b, t], r[b, t] = wp.c_kv[pg, t % s.page_size], wp.k_rope[pg, t % s.page_size]
+    wc = dataclasses.replace(wp, shape=dataclasses.replace(s, paged=False), c_kv=c, k_rope=r, block_table=None,
+                             num_pages=0, capacity=cap)
+    res = []
+    for w in (wp, wc):
+        dw = abi.to_device(w)
+        step = run_step(dw, num_splits=3)
+        res.append((step.o_lat.cpu(), step.lse.cpu(), step.o.cpu(), step.out.cpu()))
+    for a, b in zip(*res):
+        assert torch.equal(a, b)
+
+
+def test_edge_lengths():
+    """kv_len == q_len (the chunk alone), kv_len == 1, lengths ending exactly
+    on a tile boundary and one past it, and kv_len == capacity."""
+    shape = wl.SHAPES["llama1b_chunk5_b32_h32_r512_t4096"]
+    base = wl.make(shape, seed=16, batch=6, kv_range=(5, 5))
+    kv = torch.tensor([5, 6, 128, 129, 256, 300], dtype=torch.int32)
+    w = dataclasses.replace(base, kv_len=kv, start_pos=kv - 5, capacity=300,
+                            c_kv=wl._randn(torch.Generator().manual_seed(1), (6, 300, shape.rank)),
+                            k_rope=wl._randn(torch.Generator().manual_seed(2), (6, 300, shape.d_rope)))
+    dw = abi.to_device(w)
+    step = run_step(dw)
+    ref = oracle_step(w)
+    assert_close(step.o_lat.cpu().numpy(), ref["o_lat"], "o_lat")
+    assert_close(bf16_to_f64(bits(step.out.cpu())), ref["out"], "out")
+    # kv_len == 1 with q_len == 1: o_lat is exactly the single appended latent row
+    s1 = wl.SHAPES["tiny_b1_h8_r128_t256"]
+    w1 = wl.make(s1, seed=17, kv_range=(1, 1))
+    dw1 = abi.to_device(w1)
+    st1 = run_step(dw1)
+    c0 = w1.c_new[0, 0].float()
+    for h in range(s1.num_heads):
+        assert torch.equal(st1.o_lat[0, 0, h].cpu(), c0)
+
+
+def test_empty_batch_is_a_noop():
+    w = wl.small("tiny_b1_h8_r128_t256")
+    dw = abi.to_device(w)
+    empty = torch.empty(0, 1, 8, 64, dtype=torch.bfloat16, device="cuda")
+    q_abs = torch.empty(0, 1, 8, 160, dtype=torch.bfloat16, device="cuda")
+    abi.absorb_q(dw.dims, empty, empty[..., :32], dw.kv_len[:0], dw.w_uk, q_abs)
+    assert abi.check_status() == abi.MLA_OK
+
+
+def test_device_faults_are_reported_not_trapped():
+    # a block-table entry outside the page pool
+    w = wl.small("llama1b_paged_b128_h32_r512_t128_8192", seed=18)
+    w.block_table[1, 0] = w.num_pages + 7
+    dw = abi.to_device(w)
+    step = abi.DecodeStep(dw.dims, dw.cache, dw.batch, dw.q_len, dw.max_kv_len)
+    step(dw.q_nope, dw.q_pe, dw.kv_len, dw.w_uk, dw.w_uv, dw.w_o, c_new=dw.c_new, kr_new=dw.kr_new,
+         start_pos=dw.start_pos)
+    assert abi.check_status() == abi.MLA_ERR_DEVICE_BOUNDS
+    # a length above the stated maximum
+    w = wl.small("qwen05b_b16_h14_r256_t2048", seed=19)
+    dw = abi.to_device(w)
+    dw.kv_len[0] = dw.max_kv_len + 1
+    step = abi.DecodeStep(dw.dims, dw.cache, dw.batch, dw.q_len, dw.max_kv_len)
+    step(dw.q_nope, dw.q_pe, dw.kv_len, dw.w_uk, dw.w_uv, dw.w_o)
+    assert abi.check_status() == abi.MLA_ERR_DEVICE_BOUNDS
+    # an append position past the capacity
+    dw.start_pos[0] = dw.cache.capacity
+    abi.cache_append(dw.dims, dw.cache, dw.c_new, dw.kr_new, dw.start_pos)
+    assert abi.check_status() == abi.MLA_ERR_DEVICE_BOUNDS
+    # the context is still usable afterwards
+    dw = abi.to_device(wl.small("tiny_b1_h8_r128_t256"))
+    run_step(dw)
+
+
+def test_deterministic():
+    w = wl.small("llama3b_long_b8_h24_r512_t16k_32k", seed=20)
+    a = run_step(abi.to_device(w)).o_lat.cpu()
+    b = run_step(abi.to_device(w)).o_lat.cpu()
+    assert torch.equal(a, b)
