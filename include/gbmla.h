@@ -191,6 +191,11 @@ mla_status mla_check_status(void *stream);
  * with mla_check_status(). */
 mla_status mla_selftest_wait_timeout(int64_t limit_ns, void *stream);
 
+/* Text of the CUDA error behind the last MLA_ERR_CUDA returned to the calling
+ * thread ("" if none).  The library's own; it has no counterpart in the
+ * paper. */
+const char *mla_last_error(void);
+
 /* Static name of a status code. */
 const char *mla_status_str(mla_status status);
 

@@ -20,7 +20,7 @@ from . import build as _build
 MLA_OK, MLA_ERR_INVALID_ARG, MLA_ERR_UNSUPPORTED, MLA_ERR_CUDA, MLA_ERR_DEVICE_BOUNDS, MLA_ERR_DEVICE_TIMEOUT = range(6)
 SPLIT_TILE = 128
 EXPORTS = ("mla_workspace_size", "mla_cache_append", "mla_absorb_q", "mla_decode_attn", "mla_combine",
-           "mla_out_proj", "mla_check_status", "mla_selftest_wait_timeout", "mla_status_str")
+           "mla_out_proj", "mla_check_status", "mla_selftest_wait_timeout", "mla_status_str", "mla_last_error")
 
 
 class MlaError(RuntimeError):
@@ -73,7 +73,9 @@ def lib(auto_build: bool = True):
             L.mla_out_proj.argtypes = [P(MlaDims), i32, i32, vp, vp, vp, vp, vp, vp]
             L.mla_check_status.argtypes = [vp]
             L.mla_selftest_wait_timeout.argtypes = [i64, vp]
-            for name in EXPORTS[:-1]:
+            L.mla_last_error.restype = ctypes.c_char_p
+            L.mla_last_error.argtypes = []
+            for name in EXPORTS[:-2]:
                 getattr(L, name).restype = ctypes.c_int
             _lib = L
         return _lib
@@ -85,7 +87,10 @@ def status_name(code: int) -> str:
 
 def _check(where: str, code: int):
     if code != MLA_OK:
-        raise MlaError(where, code, status_name(code))
+        name = status_name(code)
+        if code == MLA_ERR_CUDA:
+            name += f" ({lib().mla_last_error().decode()})"
+        raise MlaError(where, code, name)
 
 
 def _stream(stream) -> Optional[int]:

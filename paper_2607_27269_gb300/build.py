@@ -19,7 +19,7 @@ INCLUDE = os.path.join(os.path.dirname(PKG), "include")
 BUILD_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libgbmla.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["api.cu", "append.cu", "absorb.cu", "attn_simt.cu", "combine.cu", "out_proj.cu"]
+SOURCES = ["api.cu", "append.cu", "absorb.cu", "attn_simt.cu", "attn_tc.cu", "combine.cu", "out_proj.cu"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
               "-Xptxas", "-warn-spills"] + ARCH
 

@@ -1,6 +1,8 @@
 // The C ABI of libgbmla.so (include/gbmla.h): host-side argument checks,
 // split resolution, the per-device status word and the launches.
 #include <math.h>
+#include <stdlib.h>
+#include <string.h>
 #include <mutex>
 
 #include "common.cuh"
@@ -83,22 +85,45 @@ mla_status check_cache(const mla_dims *d, const mla_cache *c, CacheView *v)
     return MLA_OK;
 }
 
+// The tensor-core kernel serves every shape with rank % 128 == 0; the
+// CUDA-core kernel serves the rest.  GBMLA_ATTN_KERNEL=simt forces the
+// CUDA-core kernel (used by tests that compare the two).
+bool use_tc_kernel(const mla_dims *d)
+{
+    const char *env = getenv("GBMLA_ATTN_KERNEL");
+    if (env && strcmp(env, "simt") == 0) return false;
+    return d->rank % 128 == 0;
+}
+
 // Partitions used for (dims, batch, q_len, max_kv_len): `requested` if > 0,
-// otherwise about two blocks per SM across the query groups, never more
+// otherwise enough partitions that the query groups fill the SMs (one CTA per
+// SM for the tensor-core kernel, two for the CUDA-core kernel), never more
 // partitions than tiles.
 int resolve_splits(const mla_dims *d, int batch, int q_len, int max_kv_len, int requested, int sms)
 {
     const int64_t max_tiles = static_cast<int64_t>(batch) * ((max_kv_len + MLA_SPLIT_TILE - 1) / MLA_SPLIT_TILE);
     if (requested > 0) return requested;
     const int rows = q_len * d->num_heads;
-    const int groups = (rows + kSimtRows - 1) / kSimtRows;
-    int64_t s = (2 * static_cast<int64_t>(sms) + groups - 1) / groups;
+    int64_t s;
+    if (use_tc_kernel(d)) {
+        s = sms / attn_tc_shape(rows).groups;  // one CTA per SM
+    } else {
+        const int groups = (rows + kSimtRows - 1) / kSimtRows;
+        s = (2 * static_cast<int64_t>(sms) + groups - 1) / groups;
+    }
     if (s > max_tiles) s = max_tiles;
     if (s < 1) s = 1;
     return static_cast<int>(s);
 }
 
-mla_status from_cuda(cudaError_t e) { return e == cudaSuccess ? MLA_OK : MLA_ERR_CUDA; }
+thread_local cudaError_t g_last_cuda_error = cudaSuccess;
+
+mla_status from_cuda(cudaError_t e)
+{
+    if (e == cudaSuccess) return MLA_OK;
+    g_last_cuda_error = e;
+    return MLA_ERR_CUDA;
+}
 
 __global__ void selftest_wait_kernel(uint64_t limit_ns, unsigned *status)
 {
@@ -195,7 +220,7 @@ mla_status mla_decode_attn(const mla_dims *dims, const mla_cache *cache, int32_t
     if (s != MLA_OK) return s;
     CacheView v;
     if ((s = check_cache(dims, cache, &v)) != MLA_OK) return s;
-    if (batch < 0 || q_len < 1 || q_len > 16 || num_splits < 0) return MLA_ERR_INVALID_ARG;
+    if (batch < 0 || q_len < 1 || q_len > 16 || num_splits < 0 || num_splits > 65535) return MLA_ERR_INVALID_ARG;
     if (max_kv_len < q_len || max_kv_len > cache->capacity) return MLA_ERR_INVALID_ARG;
     if (batch == 0) return MLA_OK;
     if (!kv_len || !q_abs || !o_part || !lse_part || !aligned16(o_part) || !aligned16(q_abs))
@@ -218,7 +243,8 @@ mla_status mla_decode_attn(const mla_dims *dims, const mla_cache *cache, int32_t
     a.lse_part = lse_part;
     a.cache = v;
     a.status = status;
-    return from_cuda(launch_attn_simt(a, static_cast<cudaStream_t>(stream)));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    return from_cuda(use_tc_kernel(dims) ? launch_attn_tc(a, st) : launch_attn_simt(a, st));
 }
 
 mla_status mla_combine(const mla_dims *dims, int32_t batch, int32_t q_len, int32_t num_splits,
@@ -268,6 +294,11 @@ mla_status mla_check_status(void *stream)
     if (word & kStatusTimeout) return MLA_ERR_DEVICE_TIMEOUT;
     if (word & kStatusBounds) return MLA_ERR_DEVICE_BOUNDS;
     return MLA_OK;
+}
+
+const char *mla_last_error(void)
+{
+    return g_last_cuda_error == cudaSuccess ? "" : cudaGetErrorString(g_last_cuda_error);
 }
 
 mla_status mla_selftest_wait_timeout(int64_t limit_ns, void *stream)

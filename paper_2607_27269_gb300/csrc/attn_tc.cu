@@ -1,0 +1,974 @@
+// Tensor-core split-KV attention core over the latent cache for sm_103a
+// (Eqs. 2-4 with the Sec. 3.3 score routing, in the absorbed form).
+//
+// One CTA = (one partition of the tile list, one group of N query rows).  Per
+// 128-token tile, with tokens on the MMA's M dimension and query rows on N:
+//     S^T [128 tok, N] = [k_rope | c] tile (K-major A) x q_abs^T (K-major B)
+//     online softmax over tokens (TMEM lane = token, column = query row)
+//     O^T [r, N]      += C^T (latent tile read as an MN-major A) x P^T
+// S^T (two buffers) and O^T live in TMEM.  The latent tile streams through a
+// ring of 64-column chunks twice, once for each product, in the order the MMA
+// warp consumes them: QK(0), QK(1), PV(0), QK(2), PV(1), ... so that the
+// softmax of tile t overlaps QK(t+1).  The second pass reads from L2.  The
+// positional keys use a buffer of their own.  With two query groups (160 query
+// rows) the two CTAs form a cluster and every cache box is multicast to both,
+// so each byte leaves L2 once per pass.
+//
+// Warp roles (448 threads): warp 0 = TMA producer, warp 1 = MMA issuer and
+// TMEM owner, warps 2..13 = softmax / epilogue (three warps per TMEM lane
+// quarter, each owning every third 16-column block of the query columns).  Every wait is bounded; a
+// wait that runs out records a timeout in the status word and the CTA winds
+// down without trapping.
+#include <cudaTypedefs.h>
+#include <math.h>
+#include <stdlib.h>
+
+#include "common.cuh"
+#include "internal.h"
+#include "tc.cuh"
+
+namespace gbmla {
+namespace {
+
+constexpr int kTile = MLA_SPLIT_TILE;     // tokens per tile (MMA M)
+constexpr int kHalf = 64;                 // tokens per TMA box (one page when paged)
+constexpr int kChunkBytes = kTile * 128;  // 128 tokens x 64 bf16 columns, SW128 K-major
+constexpr int kMaxSlots = 16;
+constexpr int kSoftmaxWarps = 12;
+constexpr int kThreads = 64 + 32 * kSoftmaxWarps;
+
+struct TcArgs {
+    int batch, q_len, heads, rank, d_rope, rows, num_splits, max_kv;
+    int paged, bt_stride, num_pages, c_slots;
+    float scale_log2;
+    const int32_t *kv_len;
+    const int32_t *block_table;
+    float *o_part, *lse_part;
+    unsigned *status;
+    uint64_t wait_ns;
+};
+
+struct __align__(8) Bars {
+    uint64_t full[kMaxSlots], empty[kMaxSlots];
+    uint64_t kr_full, kr_empty, q_full, q_free;
+    uint64_t s_full[2], s_free[2];
+    uint64_t p_full, pv_done, o_free, drain;
+    // Tail tile handshake per r-chunk m: the MMA warp (which waits on `full`
+    // in strict order) reports that chunks 2m, 2m+1 of the PV copy landed
+    // (zready); the softmax warps clear their rows past the end (zdone).
+    uint64_t zready[4], zdone[4];
+};
+
+template <int N>
+struct Shared {
+    float red[4][N];   // per TMEM-quadrant column partials
+    float m_used[N];   // exponent base of each query column (log2 domain)
+    float alpha[N];    // rescale factor of the current tile
+    float lsum[N];     // softmax denominators at the epilogue
+    int lim[N];        // last visible position of each column (-1: padding column)
+    int need_max;
+    int any_rescale;
+    int abort;         // any role gave up: producer / MMA stop issuing
+    int sm_fail;       // softmax warps gave up (read only after a named barrier)
+    uint32_t tmem_base;
+};
+
+// Tiles [t_begin, t_end) of the flattened tile list, sequence by sequence.
+struct Walk {
+    const int32_t *kv;
+    int batch, q_len, max_kv;
+    int b;
+    int64_t seq_start, nb, t, t_begin, t_end;
+
+    __device__ void init(const int32_t *kv_len, int batch_, int q_len_, int max_kv_, int64_t tb, int64_t te)
+    {
+        kv = kv_len;
+        batch = batch_;
+        q_len = q_len_;
+        max_kv = max_kv_;
+        t = tb;
+        t_begin = tb;
+        t_end = te;
+        seq_start = 0;
+        nb = 0;
+        for (b = 0; b < batch; ++b) {
+            nb = seq_tiles(kv[b], q_len, max_kv);
+            if (seq_start + nb > t) break;
+            seq_start += nb;
+        }
+    }
+    __device__ bool done() const { return t >= t_end; }
+    __device__ int tile() const { return static_cast<int>(t - seq_start); }
+    __device__ bool first() const { return t == t_begin || t == seq_start; }
+    __device__ bool last() const { return t + 1 == t_end || t + 1 == seq_start + nb; }
+    __device__ void next()
+    {
+        ++t;
+        if (t < t_end && t >= seq_start + nb) {
+            seq_start += nb;
+            for (++b; b < batch; ++b) {
+                nb = seq_tiles(kv[b], q_len, max_kv);
+                if (nb > 0) break;
+            }
+        }
+    }
+};
+
+// Where the (up to) two 64-token halves of tile j of sequence b live.
+struct TileLoc {
+    int nh;            // halves to load (1 or 2; 0 if the first page is bad)
+    int32_t tok0[2], blk[2];
+};
+
+__device__ __forceinline__ TileLoc locate(const TcArgs &a, int b, int j)
+{
+    TileLoc L;
+    const int kv = a.kv_len[b];
+    L.nh = (kv - j * kTile > kHalf) ? 2 : 1;
+    for (int h = 0; h < L.nh; ++h) {
+        if (a.paged) {
+            const int32_t pg = a.block_table[static_cast<int64_t>(b) * a.bt_stride + 2 * j + h];
+            if (pg < 0 || pg >= a.num_pages) {
+                record_status(a.status, kStatusBounds);
+                L.nh = h;
+                break;
+            }
+            L.blk[h] = pg;
+            L.tok0[h] = 0;
+        } else {
+            L.blk[h] = b;
+            L.tok0[h] = j * kTile + h * kHalf;
+        }
+    }
+    return L;
+}
+
+// A ring position: slot index and how many full passes over the ring came before.
+struct RingPos {
+    int slot, round;
+    __device__ void advance(int cs)
+    {
+        if (++slot == cs) {
+            slot = 0;
+            ++round;
+        }
+    }
+};
+
+__device__ __forceinline__ void named_sync_softmax()
+{
+    asm volatile("bar.sync 1, %0;" ::"n"(32 * kSoftmaxWarps) : "memory");
+}
+
+// Reduce 16 columns over the 32 lanes of a warp: afterwards lane l holds, in
+// v[0], the reduction of column (l % 16).
+template <int CNT, bool MAX>
+__device__ __forceinline__ void halve_step(float *v, int lane)
+{
+    const bool upper = (lane & CNT) != 0;
+#pragma unroll
+    for (int k = 0; k < CNT; ++k) {
+        const float send = upper ? v[k] : v[k + CNT];
+        const float keep = upper ? v[k + CNT] : v[k];
+        const float recv = __shfl_xor_sync(0xffffffffu, send, CNT);
+        v[k] = MAX ? fmaxf(keep, recv) : keep + recv;
+    }
+}
+
+template <bool MAX>
+__device__ __forceinline__ float reduce16(float (&v)[16], int lane)
+{
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+        const float o = __shfl_xor_sync(0xffffffffu, v[k], 16);
+        v[k] = MAX ? fmaxf(v[k], o) : v[k] + o;
+    }
+    halve_step<8, MAX>(v, lane);
+    halve_step<4, MAX>(v, lane);
+    halve_step<2, MAX>(v, lane);
+    halve_step<1, MAX>(v, lane);
+    return v[0];
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16])
+{
+    uint32_t r[16];
+    tc::ld_32x32b_x16(taddr, r);
+    tc::wait_ld();
+#pragma unroll
+    for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
+}
+
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const float (&v)[16])
+{
+    uint32_t r[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) r[j] = __float_as_uint(v[j]);
+    tc::st_32x32b_x16(taddr, r);
+    tc::wait_st();
+}
+
+// Per-thread constants of a softmax warp.
+struct SmCtx {
+    int lane, tid, quarter, half, tok, n_own, group, part, nrc, ncc, cs, n_items;
+    uint32_t lane_base, tmem, o_col0;
+    unsigned char *ring, *p_buf;
+    uint64_t lim_ns;
+    int64_t t_begin, t_end;
+};
+
+// One lane of the warp waits; a failure marks sm_fail, which the softmax
+// warps read only after their next named barrier, so they all leave together.
+template <int N>
+__device__ __forceinline__ void sm_wait(const SmCtx &c, const TcArgs &a, Shared<N> &ss, uint64_t *bar,
+                                        uint32_t parity)
+{
+    if (c.lane == 0 && !mbar_wait(smem_u32(bar), parity, c.lim_ns)) {
+        record_status(a.status, kStatusTimeout);
+        atomicOr(&ss.sm_fail, 1);
+        ss.abort = 1;
+    }
+    __syncwarp();
+}
+
+// Scores of one 16-column block in the log2 domain, masked where needed.
+template <int N>
+__device__ __forceinline__ void sm_scores(const TcArgs &a, const Shared<N> &ss, uint32_t s_base, int cb, int pos,
+                                          bool need_mask, float (&s)[16])
+{
+    tmem_ld16(s_base + cb * 16, s);
+#pragma unroll
+    for (int e = 0; e < 16; ++e) {
+        s[e] *= a.scale_log2;
+        if (need_mask && pos > ss.lim[cb * 16 + e]) s[e] = -INFINITY;
+    }
+}
+
+// Column maxima of the tile's scores over this warp's 32 tokens, into red[quarter].
+template <int N, int KOWN>
+__device__ __forceinline__ void sm_block_max(const SmCtx &c, const TcArgs &a, Shared<N> &ss, uint32_t s_base,
+                                             int pos, bool need_mask)
+{
+#pragma unroll
+    for (int ob = 0; ob < KOWN; ++ob) {
+        if (ob < c.n_own) {
+            const int cb = c.half + 3 * ob;
+            float s[16];
+            sm_scores<N>(a, ss, s_base, cb, pos, need_mask, s);
+            const float mx = reduce16<true>(s, c.lane);
+            if (c.lane < 16) ss.red[c.quarter][cb * 16 + c.lane] = mx;
+        }
+    }
+}
+
+// Normalised partial output and log-sum-exp of sequence b, whose last tile
+// in this partition was t_end_seg.
+template <int N, int KOWN>
+__device__ __forceinline__ void sm_epilogue(const SmCtx &c, const TcArgs &a, Shared<N> &ss, Bars &bars,
+                                            float (&l_part)[KOWN][16], int b, int64_t t_end_seg)
+{
+    sm_wait<N>(c, a, ss, &bars.pv_done, static_cast<uint32_t>(t_end_seg & 1));
+    named_sync_softmax();
+    if (ss.sm_fail) return;
+    tc::fence_after_sync();
+#pragma unroll
+    for (int ob = 0; ob < KOWN; ++ob) {
+        if (ob < c.n_own) {
+            const int cb = c.half + 3 * ob;
+            float v[16];
+#pragma unroll
+            for (int e = 0; e < 16; ++e) v[e] = l_part[ob][e];
+            const float ls = reduce16<false>(v, c.lane);
+            if (c.lane < 16) ss.red[c.quarter][cb * 16 + c.lane] = ls;
+        }
+    }
+    named_sync_softmax();
+    const int cc = c.tid - 64;
+    if (cc < N) {
+        const float l = ss.red[0][cc] + ss.red[1][cc] + ss.red[2][cc] + ss.red[3][cc];
+        ss.lsum[cc] = l;
+        ss.alpha[cc] = l > 0.f ? 1.f / l : 0.f;  // reused here as 1 / l
+    }
+    named_sync_softmax();
+    const int64_t slot = static_cast<int64_t>(b) + c.part;
+    const int valid_cols = a.rows - c.group * N;  // columns past it are padding
+    float *out = a.o_part + (slot * a.rows + c.group * N) * a.rank + c.tok;
+    for (int m = 0; m < c.nrc; ++m) {
+#pragma unroll
+        for (int ob = 0; ob < KOWN; ++ob) {
+            if (ob < c.n_own) {
+                const int cb = c.half + 3 * ob;
+                float o[16];
+                tmem_ld16(c.tmem + c.lane_base + c.o_col0 + m * N + cb * 16, o);
+#pragma unroll
+                for (int e = 0; e < 16; ++e) {
+                    const int col = cb * 16 + e;
+                    if (col < valid_cols) out[col * a.rank + m * 128] = o[e] * ss.alpha[col];
+                }
+            }
+        }
+    }
+    if (cc < N) {
+        const int row = c.group * N + cc;
+        if (row < a.rows) {
+            const float l = ss.lsum[cc];
+            a.lse_part[slot * a.rows + row] = l > 0.f ? (ss.m_used[cc] + log2f(l)) * 0.69314718055994531f : -INFINITY;
+        }
+    }
+    tc::fence_before_sync();
+    __syncwarp();
+    if (c.lane == 0) tc::mbar_arrive(smem_u32(&bars.o_free));
+}
+
+template <int N>
+__device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Shared<N> &ss, Bars &bars)
+{
+    constexpr int NB = N / 16;
+    constexpr int KOWN = (NB + 2) / 3;
+    float l_part[KOWN][16];
+    int b_cur = -1;
+    int64_t t_last = -1;
+    int n_tail = 0;  // tail tiles handled so far (phase of zready / zdone)
+    const int cc = c.tid - 64;
+    Walk w;
+    w.init(a.kv_len, a.batch, a.q_len, a.max_kv, c.t_begin, c.t_end);
+    for (int64_t t = 0; !w.done(); ++t, w.next()) {
+        const bool first = w.first(), last = w.last();
+        const int b = w.b, j = w.tile();
+        const int kv = a.kv_len[b];
+        const int sb = static_cast<int>(t & 1);
+        sm_wait<N>(c, a, ss, &bars.s_full[sb], static_cast<uint32_t>((t >> 1) & 1));
+        named_sync_softmax();
+        if (ss.sm_fail) break;
+        tc::fence_after_sync();
+        if (first) {
+            if (b_cur >= 0) {
+                sm_epilogue<N, KOWN>(c, a, ss, bars, l_part, b_cur, t_last);
+                if (ss.sm_fail) break;
+            }
+            b_cur = b;
+#pragma unroll
+            for (int ob = 0; ob < KOWN; ++ob)
+#pragma unroll
+                for (int e = 0; e < 16; ++e) l_part[ob][e] = 0.f;
+            if (cc < N) {
+                const int row = c.group * N + cc;
+                ss.lim[cc] = row < a.rows ? kv - a.q_len + row / a.heads : -1;
+            }
+            named_sync_softmax();
+        }
+        t_last = t;
+        const int pos = j * kTile + c.tok;
+        // the mask matters only where a token lies past the earliest query's last key
+        const bool need_mask = j * kTile + kTile - 1 > kv - a.q_len;
+        const uint32_t s_base = c.tmem + c.lane_base + sb * N;
+        // ---- pass 1: exponent bases (exact column maxima on a sequence's first
+        // tile, else only when a score passes the current base by more than 2^8)
+        if (first) {
+            sm_block_max<N, KOWN>(c, a, ss, s_base, pos, need_mask);
+            named_sync_softmax();
+            if (cc < N) {
+                ss.m_used[cc] = fmaxf(fmaxf(ss.red[0][cc], ss.red[1][cc]), fmaxf(ss.red[2][cc], ss.red[3][cc]));
+                ss.alpha[cc] = 1.f;
+            }
+            if (c.tid == 64) ss.any_rescale = 0;
+        } else {
+            bool over = false;
+#pragma unroll
+            for (int ob = 0; ob < KOWN; ++ob) {
+                if (ob < c.n_own) {
+                    const int cb = c.half + 3 * ob;
+                    float s[16];
+                    sm_scores<N>(a, ss, s_base, cb, pos, need_mask, s);
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) over |= s[e] > ss.m_used[cb * 16 + e] + 8.f;
+                }
+            }
+            if (__any_sync(0xffffffffu, over) && c.lane == 0) ss.need_max = 1;
+            named_sync_softmax();
+            if (ss.need_max) {  // uniform: written before the barrier, read after it
+                sm_block_max<N, KOWN>(c, a, ss, s_base, pos, need_mask);
+                named_sync_softmax();
+                if (cc < N) {
+                    const float tmax = fmaxf(fmaxf(ss.red[0][cc], ss.red[1][cc]), fmaxf(ss.red[2][cc], ss.red[3][cc]));
+                    const float m_old = ss.m_used[cc];
+                    float alpha = 1.f;
+                    if (tmax != -INFINITY && (m_old == -INFINITY || tmax > m_old + 8.f)) {
+                        alpha = m_old == -INFINITY ? 0.f : exp2f(m_old - tmax);
+                        ss.m_used[cc] = tmax;
+                    }
+                    ss.alpha[cc] = alpha;
+                }
+                if (c.tid == 64) {
+                    ss.any_rescale = 1;
+                    ss.need_max = 0;
+                }
+            } else if (c.tid == 64) {
+                ss.any_rescale = 0;
+            }
+        }
+        named_sync_softmax();
+        // ---- P is rewritten and O^T rescaled only once PV(t-1) has completed
+        if (!first) {
+            sm_wait<N>(c, a, ss, &bars.pv_done, static_cast<uint32_t>((t - 1) & 1));
+            named_sync_softmax();
+            if (ss.sm_fail) break;
+            tc::fence_after_sync();
+            if (ss.any_rescale) {
+#pragma unroll
+                for (int ob = 0; ob < KOWN; ++ob) {
+                    if (ob < c.n_own) {
+                        const int cb = c.half + 3 * ob;
+                        float al[16];
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) {
+                            al[e] = ss.alpha[cb * 16 + e];
+                            l_part[ob][e] *= al[e];
+                        }
+                        for (int m = 0; m < c.nrc; ++m) {
+                            const uint32_t ta = c.tmem + c.lane_base + c.o_col0 + m * N + cb * 16;
+                            float o[16];
+                            tmem_ld16(ta, o);
+#pragma unroll
+                            for (int e = 0; e < 16; ++e) o[e] *= al[e];
+                            tmem_st16(ta, o);
+                        }
+                    }
+                }
+            }
+        }
+        // ---- pass 2: P = 2^(s - m) in bf16 (MN-major, 16-column SW32 atoms), running sums
+#pragma unroll
+        for (int ob = 0; ob < KOWN; ++ob) {
+            if (ob < c.n_own) {
+                const int cb = c.half + 3 * ob;
+                float s[16];
+                sm_scores<N>(a, ss, s_base, cb, pos, need_mask, s);
+                uint32_t pk[8];
+#pragma unroll
+                for (int e = 0; e < 16; e += 2) {
+                    const float p0 = s[e] == -INFINITY ? 0.f : exp2f(s[e] - ss.m_used[cb * 16 + e]);
+                    const float p1 = s[e + 1] == -INFINITY ? 0.f : exp2f(s[e + 1] - ss.m_used[cb * 16 + e + 1]);
+                    const __nv_bfloat162 pb = __floats2bfloat162_rn(p0, p1);
+                    l_part[ob][e] += __low2float(pb);  // the weights the MMA multiplies by
+                    l_part[ob][e + 1] += __high2float(pb);
+                    pk[e / 2] = *reinterpret_cast<const uint32_t *>(&pb);
+                }
+                unsigned char *row = c.p_buf + cb * (kTile * 32) + c.tok * 32;
+                const int sw = (c.tok >> 2) & 1;
+                *reinterpret_cast<uint4 *>(row + (sw * 16)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                *reinterpret_cast<uint4 *>(row + ((1 ^ sw) * 16)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+            }
+        }
+        tc::fence_before_sync();
+        __syncwarp();
+        if (c.lane == 0) tc::mbar_arrive(smem_u32(&bars.s_free[sb]));
+        tc::fence_proxy_async_smem();
+        tc::fence_before_sync();
+        __syncwarp();
+        if (c.lane == 0) tc::mbar_arrive(smem_u32(&bars.p_full));
+        // ---- tail tile: rows past the sequence end in the PV copy of the
+        // latent chunks are cleared, so stale or uninitialised bytes never meet
+        // a zero weight.  P is already published; the MMA warp reports each
+        // landed pair (zready) and waits for it to be cleared (zdone), so every
+        // wait here is on the next phase of its barrier.
+        if (last && kv - j * kTile < kTile) {
+            const int64_t qk_groups = (t + 2 < c.n_items) ? t + 2 : c.n_items;
+            const int64_t g0 = static_cast<int64_t>(c.ncc) * (qk_groups + t);
+            for (int m = 0; m < c.nrc; ++m) {
+                sm_wait<N>(c, a, ss, &bars.zready[m], static_cast<uint32_t>(n_tail & 1));
+                if (pos >= kv) {
+                    for (int k = 0; k < 2; ++k) {
+                        const int slot = static_cast<int>((g0 + 2 * m + k) % c.cs);
+                        // three warps share a quarter's rows: 16-byte pieces half, half+3, ...
+                        uint4 *dst = reinterpret_cast<uint4 *>(c.ring + slot * kChunkBytes + c.tok * 128);
+                        for (int q = c.half; q < 8; q += 3) dst[q] = make_uint4(0, 0, 0, 0);
+                    }
+                }
+                tc::fence_proxy_async_smem();
+                __syncwarp();
+                if (c.lane == 0) tc::mbar_arrive(smem_u32(&bars.zdone[m]));
+            }
+            ++n_tail;
+        }
+    }
+    named_sync_softmax();
+    if (b_cur >= 0 && !ss.sm_fail) sm_epilogue<N, KOWN>(c, a, ss, bars, l_part, b_cur, t_last);
+}
+
+// N: query rows per CTA (multiple of 16, <= 80).  CL: CTAs per cluster (1 or 2).
+template <int N, int CL>
+__global__ void __maxnreg__(128)
+    attn_tc_kernel(const __grid_constant__ TcArgs a, const __grid_constant__ CUtensorMap map_c,
+                   const __grid_constant__ CUtensorMap map_r, const __grid_constant__ CUtensorMap map_q)
+{
+    constexpr int NB = N / 16;                   // 16-column blocks
+    constexpr uint16_t kMask = (1u << CL) - 1;
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    __shared__ Bars bars;
+    __shared__ Shared<N> ss;
+    __shared__ int64_t red64[32];
+
+    unsigned char *smem = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                            ~static_cast<uintptr_t>(1023));
+    const int ncc = a.rank / 64;    // latent chunks per tile
+    const int nrc = a.rank / 128;   // r-chunks of O^T
+    const int CS = a.c_slots;       // ring slots (even)
+    unsigned char *q_buf = smem;                                                // (ncc+1) x [N x 128 B]
+    unsigned char *kr_buf = q_buf + (((ncc + 1) * N * 128 + 1023) & ~1023);     // [128 x 128 B]
+    unsigned char *ring = kr_buf + kChunkBytes;                                 // CS x [128 x 128 B]
+    unsigned char *p_buf = ring + CS * kChunkBytes;                             // NB x [128 tok x 32 B]
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int group = blockIdx.x, part = blockIdx.y;
+    const uint32_t rank_in_cluster = CL > 1 ? tc::cluster_ctarank() : 0;
+    const uint64_t lim_ns = a.wait_ns;
+
+    if (part == 0 && group == 0) {
+        for (int bb = tid; bb < a.batch; bb += kThreads) {
+            const int kv = a.kv_len[bb];
+            if (kv < a.q_len || kv > a.max_kv) record_status(a.status, kStatusBounds);
+        }
+    }
+    const int64_t T = block_tile_sum(a.kv_len, a.batch, a.q_len, a.max_kv, red64);
+    const int64_t t_begin = T ? part_begin(part, T, a.num_splits) : 0;
+    const int64_t t_end = T ? part_begin(part + 1, T, a.num_splits) : 0;
+    const int n_items = static_cast<int>(t_end - t_begin);
+
+    if (tid == 0) {
+        for (int i = 0; i < kMaxSlots; ++i) {
+            mbar_init(&bars.full[i], 1);
+            mbar_init(&bars.empty[i], CL);
+        }
+        mbar_init(&bars.kr_full, 1);
+        mbar_init(&bars.kr_empty, CL);
+        mbar_init(&bars.q_full, 1);
+        mbar_init(&bars.q_free, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&bars.s_full[i], 1);
+            mbar_init(&bars.s_free[i], kSoftmaxWarps);
+        }
+        mbar_init(&bars.p_full, kSoftmaxWarps);
+        mbar_init(&bars.pv_done, 1);
+        mbar_init(&bars.o_free, kSoftmaxWarps);
+        mbar_init(&bars.drain, 1);
+        for (int i = 0; i < 4; ++i) {
+            mbar_init(&bars.zready[i], 1);
+            mbar_init(&bars.zdone[i], kSoftmaxWarps);
+        }
+        ss.need_max = 0;
+        ss.any_rescale = 0;
+        ss.abort = 0;
+        ss.sm_fail = 0;
+        tc::fence_barrier_init();
+    }
+    if (warp == 1) {
+        constexpr uint32_t cols = (2 * N + 4 * N) <= 128 ? 128 : ((2 * N + 4 * N) <= 256 ? 256 : 512);
+        tc::tmem_alloc(smem_u32(&ss.tmem_base), cols);
+        tc::tmem_relinquish();
+    }
+    tc::fence_before_sync();
+    __syncthreads();
+    if (CL > 1) tc::cluster_sync();  // peers may multicast into this CTA only after its barriers exist
+    tc::fence_after_sync();
+    const uint32_t tmem = ss.tmem_base;
+    const uint32_t o_col0 = 2 * N;   // S^T buffers at columns [0, N) and [N, 2N)
+
+    if (warp == 0) {
+        // ================================================================ TMA producer
+        if (lane == 0 && n_items > 0) {
+            tc::prefetch_tensormap(&map_c);
+            tc::prefetch_tensormap(&map_r);
+            tc::prefetch_tensormap(&map_q);
+            Walk wq, wp;
+            wq.init(a.kv_len, a.batch, a.q_len, a.max_kv, t_begin, t_end);
+            wp.init(a.kv_len, a.batch, a.q_len, a.max_kv, t_begin, t_end);
+            RingPos rp{0, 0};
+            int kr_uses = 0, seg = -1;
+            int64_t chunk_no = 0;
+            bool ok = true;
+            auto load_chunks = [&](const TileLoc &L) {
+                const uint32_t bytes = static_cast<uint32_t>(L.nh) * kHalf * 128;
+                for (int i = 0; i < ncc && ok; ++i) {
+                    if (rp.round >= 1 && !mbar_wait(smem_u32(&bars.empty[rp.slot]), (rp.round - 1) & 1, lim_ns)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t full = smem_u32(&bars.full[rp.slot]);
+                    tc::mbar_arrive_expect_tx(full, bytes);
+                    if (chunk_no % CL == rank_in_cluster) {
+                        const uint32_t dst = smem_u32(ring + rp.slot * kChunkBytes);
+                        for (int h = 0; h < L.nh; ++h) {
+                            if (CL > 1)
+                                tc::tma_load_3d_multicast(dst + h * kHalf * 128, &map_c, 64 * i, L.tok0[h], L.blk[h],
+                                                          full, kMask);
+                            else
+                                tc::tma_load_3d(dst + h * kHalf * 128, &map_c, 64 * i, L.tok0[h], L.blk[h], full);
+                        }
+                    }
+                    ++chunk_no;
+                    rp.advance(CS);
+                }
+            };
+            auto emit_qk = [&]() {
+                const int b = wq.b, j = wq.tile();
+                if (wq.first()) {
+                    ++seg;
+                    if (seg >= 1 && !mbar_wait(smem_u32(&bars.q_free), (seg - 1) & 1, lim_ns)) {
+                        ok = false;
+                        return;
+                    }
+                    tc::mbar_arrive_expect_tx(smem_u32(&bars.q_full), (ncc + 1) * N * 128);
+                    for (int i = 0; i <= ncc; ++i)
+                        tc::tma_load_2d(smem_u32(q_buf + i * N * 128), &map_q, 64 * i, b * a.rows + group * N,
+                                        smem_u32(&bars.q_full));
+                }
+                const TileLoc L = locate(a, b, j);
+                if (kr_uses >= 1 && !mbar_wait(smem_u32(&bars.kr_empty), (kr_uses - 1) & 1, lim_ns)) {
+                    ok = false;
+                    return;
+                }
+                const uint32_t krf = smem_u32(&bars.kr_full);
+                tc::mbar_arrive_expect_tx(krf, static_cast<uint32_t>(L.nh) * kHalf * 128);
+                if (kr_uses % CL == static_cast<int>(rank_in_cluster)) {
+                    for (int h = 0; h < L.nh; ++h) {
+                        if (CL > 1)
+                            tc::tma_load_3d_multicast(smem_u32(kr_buf) + h * kHalf * 128, &map_r, 0, L.tok0[h],
+                                                      L.blk[h], krf, kMask);
+                        else
+                            tc::tma_load_3d(smem_u32(kr_buf) + h * kHalf * 128, &map_r, 0, L.tok0[h], L.blk[h], krf);
+                    }
+                }
+                ++kr_uses;
+                load_chunks(L);
+                wq.next();
+            };
+            auto emit_pv = [&]() {
+                load_chunks(locate(a, wp.b, wp.tile()));
+                wp.next();
+            };
+            emit_qk();
+            for (int t = 0; t < n_items && ok && !*reinterpret_cast<volatile int *>(&ss.abort); ++t) {
+                if (t + 1 < n_items) emit_qk();
+                if (!ok) break;
+                emit_pv();
+            }
+            if (!ok) {
+                record_status(a.status, kStatusTimeout);
+                ss.abort = 1;
+            }
+        }
+    } else if (warp == 1) {
+        // ================================================================ MMA issuer
+        if (lane == 0 && n_items > 0) {
+            const uint32_t id_qk = tc::idesc_bf16_f32(128, N, false, false);
+            const uint32_t id_pv = tc::idesc_bf16_f32(128, N, true, true);
+            const uint32_t q_base = smem_u32(q_buf), kr_base = smem_u32(kr_buf);
+            const uint32_t ring_base = smem_u32(ring), p_base = smem_u32(p_buf);
+            // descriptor templates (start address added per MMA)
+            const uint64_t dq = tc::smem_desc(0, 16, 1024, tc::kSwizzle128B);
+            const uint64_t dc = tc::smem_desc(0, kChunkBytes, 1024, tc::kSwizzle128B);
+            const uint64_t dp = tc::smem_desc(0, 128 * 32, 256, tc::kSwizzle32B);
+            auto with_addr = [](uint64_t tmpl, uint32_t saddr) {
+                return tmpl | static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+            };
+            Walk wq, wp;
+            wq.init(a.kv_len, a.batch, a.q_len, a.max_kv, t_begin, t_end);
+            wp.init(a.kv_len, a.batch, a.q_len, a.max_kv, t_begin, t_end);
+            RingPos rp{0, 0};
+            int kr_uses = 0, seg_q = -1, seg_p = -1, tq = 0, n_tail = 0;
+            bool ok = true;
+            auto wait = [&](uint64_t *bar, uint32_t parity) {
+                if (ok && !mbar_wait(smem_u32(bar), parity, lim_ns)) ok = false;
+                return ok;
+            };
+            // a consumed slot is handed back to every CTA of the cluster
+            auto release = [&](uint64_t *bar) {
+                if (CL > 1)
+                    tc::commit_multicast(smem_u32(bar), kMask);
+                else
+                    tc::commit(smem_u32(bar));
+            };
+            auto do_qk = [&]() {
+                if (wq.first()) {
+                    ++seg_q;
+                    if (!wait(&bars.q_full, seg_q & 1)) return;
+                }
+                const int sb = tq & 1;
+                if (tq >= 2 && !wait(&bars.s_free[sb], ((tq >> 1) - 1) & 1)) return;
+                if (!wait(&bars.kr_full, kr_uses & 1)) return;
+                tc::fence_after_sync();
+                const uint32_t d_s = tmem + sb * N;
+                const uint32_t qr = q_base + ncc * N * 128;
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+                    tc::mma_bf16(d_s, with_addr(dq, kr_base + k * 32), with_addr(dq, qr + k * 32), id_qk, k > 0);
+                release(&bars.kr_empty);
+                ++kr_uses;
+                for (int i = 0; i < ncc; ++i) {
+                    if (!wait(&bars.full[rp.slot], rp.round & 1)) return;
+                    tc::fence_after_sync();
+                    const uint32_t cb = ring_base + rp.slot * kChunkBytes;
+                    const uint32_t qb = q_base + i * N * 128;
+#pragma unroll
+                    for (int k = 0; k < 4; ++k)
+                        tc::mma_bf16(d_s, with_addr(dq, cb + k * 32), with_addr(dq, qb + k * 32), id_qk, 1);
+                    release(&bars.empty[rp.slot]);
+                    rp.advance(CS);
+                }
+                tc::commit(smem_u32(&bars.s_full[sb]));
+                if (wq.last()) tc::commit(smem_u32(&bars.q_free));
+                ++tq;
+                wq.next();
+            };
+            auto do_pv = [&](int t) {
+                if (!wait(&bars.p_full, t & 1)) return;
+                bool first_pv = false;
+                if (wp.first()) {
+                    ++seg_p;
+                    if (seg_p >= 1 && !wait(&bars.o_free, (seg_p - 1) & 1)) return;
+                    first_pv = true;
+                }
+                // a sequence's last, partial tile: its rows past the end are cleared
+                // by the softmax warps, pair by pair, before PV reads them
+                const bool tail = wp.last() && a.kv_len[wp.b] - wp.tile() * kTile < kTile;
+                for (int m = 0; m < nrc; ++m) {
+                    // chunks 2m, 2m+1 sit in adjacent slots (every group starts at an even slot)
+                    const int s0 = rp.slot;
+                    if (!wait(&bars.full[s0], rp.round & 1) || !wait(&bars.full[s0 + 1], rp.round & 1)) return;
+                    if (tail) {
+                        tc::mbar_arrive(smem_u32(&bars.zready[m]));
+                        if (!wait(&bars.zdone[m], n_tail & 1)) return;
+                    }
+                    tc::fence_after_sync();
+                    const uint32_t cb = ring_base + s0 * kChunkBytes;
+                    const uint32_t d_o = tmem + o_col0 + m * N;
+#pragma unroll
+                    for (int kk = 0; kk < kTile / 16; ++kk)
+                        tc::mma_bf16(d_o, with_addr(dc, cb + kk * 16 * 128), with_addr(dp, p_base + kk * 16 * 32), id_pv,
+                                     (first_pv && kk == 0) ? 0u : 1u);
+                    release(&bars.empty[s0]);
+                    release(&bars.empty[s0 + 1]);
+                    rp.advance(CS);
+                    rp.advance(CS);
+                }
+                tc::commit(smem_u32(&bars.pv_done));
+                if (tail) ++n_tail;
+                wp.next();
+            };
+            do_qk();
+            for (int t = 0; t < n_items && ok && !*reinterpret_cast<volatile int *>(&ss.abort); ++t) {
+                if (t + 1 < n_items) do_qk();
+                if (!ok) break;
+                do_pv(t);
+            }
+            if (!ok) {
+                record_status(a.status, kStatusTimeout);
+                ss.abort = 1;
+            }
+            // drain: every MMA this thread issued has completed before TMEM is freed
+            tc::commit(smem_u32(&bars.drain));
+            if (!mbar_wait(smem_u32(&bars.drain), 0, lim_ns)) record_status(a.status, kStatusTimeout);
+        }
+    } else {
+        // ================================================================ softmax / epilogue
+        SmCtx c;
+        c.lane = lane;
+        c.tid = tid;
+        c.quarter = warp & 3;                 // TMEM lane quarter this warp may access
+        c.half = (warp - 2) >> 2;             // which column blocks it owns: half, half+3, ...
+        c.tok = c.quarter * 32 + lane;        // token row of the tile
+        c.n_own = c.half < NB ? (NB - c.half + 2) / 3 : 0;
+        c.group = group;
+        c.part = part;
+        c.nrc = nrc;
+        c.ncc = ncc;
+        c.cs = CS;
+        c.n_items = n_items;
+        c.lane_base = static_cast<uint32_t>(c.quarter * 32) << 16;
+        c.tmem = tmem;
+        c.o_col0 = o_col0;
+        c.ring = ring;
+        c.p_buf = p_buf;
+        c.lim_ns = lim_ns;
+        c.t_begin = t_begin;
+        c.t_end = t_end;
+        softmax_role<N>(c, a, ss, bars);
+    }
+
+    tc::fence_before_sync();
+    __syncthreads();
+    if (CL > 1) tc::cluster_sync();  // no CTA leaves while a peer may still signal it
+    if (warp == 1) {
+        tc::fence_after_sync();
+        constexpr uint32_t cols = (2 * N + 4 * N) <= 128 ? 128 : ((2 * N + 4 * N) <= 256 ? 256 : 512);
+        tc::tmem_dealloc(tmem, cols);
+    }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+cudaError_t get_encoder()
+{
+    if (g_encode) return cudaSuccess;
+    cudaDriverEntryPointQueryResult q;
+    void *fn = nullptr;
+    cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn) return e != cudaSuccess ? e : cudaErrorNotSupported;
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    return cudaSuccess;
+}
+
+// 3-d map over one cache: (columns, tokens per block, blocks), box 64 x 64 x 1, SW128.
+cudaError_t encode_cache_map(CUtensorMap *m, const void *base, int cols, int64_t tok_stride, int64_t blk_stride,
+                             int tokens_per_block, int blocks)
+{
+    cuuint64_t dims[3] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(tokens_per_block),
+                          static_cast<cuuint64_t>(blocks)};
+    cuuint64_t strides[2] = {static_cast<cuuint64_t>(tok_stride) * 2, static_cast<cuuint64_t>(blk_stride) * 2};
+    cuuint32_t box[3] = {64, static_cast<cuuint32_t>(kHalf), 1};
+    cuuint32_t es[3] = {1, 1, 1};
+    CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, es,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+template <int N, int CL>
+cudaError_t launch_cfg(const AttnArgs &a, int groups, cudaStream_t st)
+{
+    cudaError_t e = get_encoder();
+    if (e != cudaSuccess) return e;
+    const CacheView &c = a.cache;
+    const bool paged = c.block_table != nullptr;
+    const int tpb = paged ? c.page_size : c.capacity;
+    const int blocks = paged ? c.num_pages : a.batch;
+    CUtensorMap mc, mr, mq;
+    if ((e = encode_cache_map(&mc, c.c_kv, a.rank, c.c_tok, c.c_blk, tpb, blocks)) != cudaSuccess) return e;
+    if ((e = encode_cache_map(&mr, c.k_rope, a.d_rope, c.r_tok, c.r_blk, tpb, blocks)) != cudaSuccess) return e;
+    {
+        const int K = a.rank + a.d_rope;
+        cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(a.batch) * a.q_len * a.num_heads};
+        cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
+        cuuint32_t box[2] = {64, N};
+        cuuint32_t es[2] = {1, 1};
+        CUresult r = g_encode(&mq, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(a.q_abs), dims, strides,
+                              box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    }
+    const int ncc = a.rank / 64;
+    const int q_bytes = (((ncc + 1) * N * 128) + 1023) & ~1023;
+    const int p_bytes = (N / 16) * kTile * 32;
+    const int fixed = 1024 /*alignment slack*/ + q_bytes + kChunkBytes /*positional keys*/;
+    int dev = 0, optin = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    const int static_bytes = static_cast<int>(sizeof(Bars) + sizeof(Shared<N>) + 32 * 8) + 128;
+    int slots = (optin - static_bytes - fixed - p_bytes) / kChunkBytes;
+    if (slots > kMaxSlots) slots = kMaxSlots;
+    if (const char *env = getenv("GBMLA_TC_MAX_SLOTS")) {  // testing aid: a smaller ring
+        const int cap = atoi(env);
+        if (cap >= 4 && cap < slots) slots = cap;
+    }
+    slots &= ~1;
+    if (slots < 4) return cudaErrorInvalidConfiguration;
+    const size_t smem = static_cast<size_t>(fixed) + static_cast<size_t>(slots) * kChunkBytes + p_bytes;
+    if ((e = cudaFuncSetAttribute(attn_tc_kernel<N, CL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  static_cast<int>(smem))) != cudaSuccess)
+        return e;
+    TcArgs t;
+    t.batch = a.batch;
+    t.q_len = a.q_len;
+    t.heads = a.num_heads;
+    t.rank = a.rank;
+    t.d_rope = a.d_rope;
+    t.rows = a.q_len * a.num_heads;
+    t.num_splits = a.num_splits;
+    t.max_kv = a.max_kv;
+    t.paged = paged;
+    t.bt_stride = c.bt_stride;
+    t.num_pages = c.num_pages;
+    t.c_slots = slots;
+    t.scale_log2 = a.sm_scale * 1.4426950408889634f;
+    t.kv_len = a.kv_len;
+    t.block_table = c.block_table;
+    t.o_part = a.o_part;
+    t.lse_part = a.lse_part;
+    t.status = a.status;
+    t.wait_ns = kWaitLimitNs;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(groups, a.num_splits, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    if (CL > 1) {
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = CL;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+    }
+    return cudaLaunchKernelEx(&cfg, attn_tc_kernel<N, CL>, t, mc, mr, mq);
+}
+
+}  // namespace
+
+TcShape attn_tc_shape(int rows)
+{
+    // Testing aids, read at every call: GBMLA_TC_MAX_N caps the query rows per
+    // CTA (16..80), GBMLA_TC_NO_CLUSTER=1 runs two query groups as separate
+    // CTAs (each loading the cache itself) instead of a multicast cluster.
+    int max_n = 80;
+    if (const char *e = getenv("GBMLA_TC_MAX_N")) max_n = atoi(e);
+    if (max_n < 16) max_n = 16;
+    if (max_n > 80) max_n = 80;
+    max_n -= max_n % 16;
+    const bool no_cluster = getenv("GBMLA_TC_NO_CLUSTER") != nullptr;
+    TcShape s;
+    if (max_n < 80) {
+        s.groups = (rows + max_n - 1) / max_n;
+        s.n = (((rows + s.groups - 1) / s.groups + 15) / 16) * 16;
+        s.cluster = 1;
+        return s;
+    }
+    if (rows <= 80) {
+        s.n = ((rows + 15) / 16) * 16;
+        s.groups = 1;
+        s.cluster = 1;
+    } else if (rows <= 160) {
+        s.n = (((rows + 1) / 2 + 15) / 16) * 16;
+        s.groups = 2;
+        s.cluster = no_cluster ? 1 : 2;
+    } else {
+        s.n = 80;
+        s.groups = (rows + 79) / 80;
+        s.cluster = 1;
+    }
+    return s;
+}
+
+cudaError_t launch_attn_tc(const AttnArgs &a, cudaStream_t st)
+{
+    const TcShape s = attn_tc_shape(a.q_len * a.num_heads);
+    if (s.cluster == 2) {
+        switch (s.n) {
+        case 48: return launch_cfg<48, 2>(a, s.groups, st);
+        case 64: return launch_cfg<64, 2>(a, s.groups, st);
+        case 80: return launch_cfg<80, 2>(a, s.groups, st);
+        default: return cudaErrorInvalidConfiguration;
+        }
+    }
+    switch (s.n) {
+    case 16: return launch_cfg<16, 1>(a, s.groups, st);
+    case 32: return launch_cfg<32, 1>(a, s.groups, st);
+    case 48: return launch_cfg<48, 1>(a, s.groups, st);
+    case 64: return launch_cfg<64, 1>(a, s.groups, st);
+    case 80: return launch_cfg<80, 1>(a, s.groups, st);
+    default: return cudaErrorInvalidConfiguration;
+    }
+}
+
+}  // namespace gbmla

@@ -41,6 +41,15 @@ cudaError_t launch_absorb(const mla_dims &d, int batch, int q_len, const void *q
 constexpr int kSimtRows = 16;
 cudaError_t launch_attn_simt(const AttnArgs &a, cudaStream_t st);
 
+// Tensor-core attention core (tcgen05 + TMA).  For q_len * num_heads query
+// rows it runs `groups` CTAs of `n` rows per partition; with cluster == 2 the
+// two groups share every cache load through multicast.
+struct TcShape {
+    int n, groups, cluster;
+};
+TcShape attn_tc_shape(int rows);
+cudaError_t launch_attn_tc(const AttnArgs &a, cudaStream_t st);
+
 cudaError_t launch_combine(int batch, int q_len, int num_heads, int rank, int max_kv, int num_splits,
                            const int32_t *kv_len, const float *o_part, const float *lse_part, float *o_lat,
                            float *lse, cudaStream_t st);
