@@ -179,6 +179,30 @@ mla_status mla_combine(const mla_dims *dims, int32_t batch, int32_t q_len, int32
 mla_status mla_out_proj(const mla_dims *dims, int32_t batch, int32_t q_len, const float *o_lat,
                         const void *w_uv, const void *w_o, void *o, void *out, void *stream);
 
+/* mla_decode_attn followed by mla_combine, for callers that cannot allocate
+ * device memory: code that runs where an allocation is not allowed (inside a
+ * runtime that owns all device memory through its own pool, in an inference
+ * path whose memory budget is fixed up front, or in a plugin handed only its
+ * input and output tensors).  It allocates nothing and takes no partial
+ * buffers: the split partials go to one array of 32 MiB that the library
+ * reserves statically on every device that loads it, for the life of the
+ * process.  The paper has no counterpart; this is a property of the library.
+ *   Inputs as for mla_decode_attn; outputs o_lat [batch, q_len, H, rank] fp32
+ *   and lse [batch, q_len, H] fp32 (or NULL), as mla_combine writes them.
+ *   num_splits > 0 is used as given; 0 picks the usual automatic count,
+ *   lowered if needed so that (batch + S - 1) * q_len * H * (rank + 1) floats
+ *   fit the array.  A size that cannot fit returns MLA_ERR_UNSUPPORTED
+ *   before anything is launched.
+ *   The first call on a device looks up the array's device address with that
+ *   device current (a host-side query); make that first call before any stream
+ *   capture.  Every call uses the same array, so calls that overlap on the GPU
+ *   (different streams, or different threads) race and must be serialised;
+ *   each call writes every partial it later reads, so nothing has to start at
+ *   zero and stale contents from an earlier call are never used. */
+mla_status mla_decode_attn_noalloc(const mla_dims *dims, const mla_cache *cache, int32_t batch, int32_t q_len,
+                                   const int32_t *kv_len, int32_t max_kv_len, const void *q_abs, int32_t num_splits,
+                                   float *o_lat, float *lse, void *stream);
+
 /* Synchronise `stream`, then read and clear the current device's sticky
  * status word: MLA_OK, MLA_ERR_DEVICE_BOUNDS or MLA_ERR_DEVICE_TIMEOUT
  * (MLA_ERR_CUDA if the synchronisation itself failed). */

@@ -20,7 +20,8 @@ from . import build as _build
 MLA_OK, MLA_ERR_INVALID_ARG, MLA_ERR_UNSUPPORTED, MLA_ERR_CUDA, MLA_ERR_DEVICE_BOUNDS, MLA_ERR_DEVICE_TIMEOUT = range(6)
 SPLIT_TILE = 128
 EXPORTS = ("mla_workspace_size", "mla_cache_append", "mla_absorb_q", "mla_decode_attn", "mla_combine",
-           "mla_out_proj", "mla_check_status", "mla_selftest_wait_timeout", "mla_status_str", "mla_last_error")
+           "mla_out_proj", "mla_check_status", "mla_selftest_wait_timeout", "mla_decode_attn_noalloc",
+           "mla_status_str", "mla_last_error")
 
 
 class MlaError(RuntimeError):
@@ -73,6 +74,7 @@ def lib(auto_build: bool = True):
             L.mla_out_proj.argtypes = [P(MlaDims), i32, i32, vp, vp, vp, vp, vp, vp]
             L.mla_check_status.argtypes = [vp]
             L.mla_selftest_wait_timeout.argtypes = [i64, vp]
+            L.mla_decode_attn_noalloc.argtypes = [P(MlaDims), P(MlaCache), i32, i32, vp, i32, vp, i32, vp, vp, vp]
             L.mla_last_error.restype = ctypes.c_char_p
             L.mla_last_error.argtypes = []
             for name in EXPORTS[:-2]:
@@ -192,6 +194,16 @@ def out_proj(dims: Dims, o_lat: torch.Tensor, w_uv: torch.Tensor, w_o: Optional[
     batch, q_len = o_lat.shape[0], o_lat.shape[1]
     _check("mla_out_proj", lib().mla_out_proj(ctypes.byref(dims.c()), batch, q_len, _p(o_lat), _p(w_uv), _p(w_o),
                                               _p(o), _p(out), _stream(stream)))
+
+
+def decode_attn_noalloc(dims: Dims, cache: Cache, kv_len: torch.Tensor, max_kv_len: int, q_abs: torch.Tensor,
+                        o_lat: torch.Tensor, lse: Optional[torch.Tensor] = None, num_splits: int = 0, stream=None):
+    """Attention core and combine with the library's static scratch (for callers
+    that cannot allocate device memory): writes o_lat and lse directly."""
+    batch, q_len = q_abs.shape[0], q_abs.shape[1]
+    _check("mla_decode_attn_noalloc",
+           lib().mla_decode_attn_noalloc(ctypes.byref(dims.c()), ctypes.byref(cache.c()), batch, q_len, _p(kv_len),
+                                         max_kv_len, _p(q_abs), num_splits, _p(o_lat), _p(lse), _stream(stream)))
 
 
 def check_status(stream=None) -> int:

@@ -118,6 +118,34 @@ int resolve_splits(const mla_dims *d, int batch, int q_len, int max_kv_len, int 
 
 thread_local cudaError_t g_last_cuda_error = cudaSuccess;
 
+// Scratch of mla_decode_attn_noalloc: the split partials live here instead of
+// in caller buffers.  32 MiB, reserved on every device that loads the library
+// for as long as the process lives.  Host code cannot use the symbol's name as
+// a device address; noalloc_scratch() looks the address up per device.
+constexpr size_t kNoallocScratchFloats = (size_t{32} << 20) / sizeof(float);
+static __device__ __align__(256) float g_noalloc_scratch[kNoallocScratchFloats];
+float *g_noalloc_ptr[kMaxDevices];
+
+// Device address of this device's scratch array, looked up once per device
+// with that device current (a host-side query; nothing is allocated).
+mla_status noalloc_scratch(float **out)
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return MLA_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(g_mutex);
+    if (!g_noalloc_ptr[dev]) {
+        void *p = nullptr;
+        const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess) {
+            g_last_cuda_error = e;
+            return MLA_ERR_CUDA;
+        }
+        g_noalloc_ptr[dev] = static_cast<float *>(p);
+    }
+    *out = g_noalloc_ptr[dev];
+    return MLA_OK;
+}
+
 mla_status from_cuda(cudaError_t e)
 {
     if (e == cudaSuccess) return MLA_OK;
@@ -294,6 +322,63 @@ mla_status mla_check_status(void *stream)
     if (word & kStatusTimeout) return MLA_ERR_DEVICE_TIMEOUT;
     if (word & kStatusBounds) return MLA_ERR_DEVICE_BOUNDS;
     return MLA_OK;
+}
+
+mla_status mla_decode_attn_noalloc(const mla_dims *dims, const mla_cache *cache, int32_t batch, int32_t q_len,
+                                   const int32_t *kv_len, int32_t max_kv_len, const void *q_abs, int32_t num_splits,
+                                   float *o_lat, float *lse, void *stream)
+{
+    mla_status s = check_dims(dims);
+    if (s != MLA_OK) return s;
+    CacheView v;
+    if ((s = check_cache(dims, cache, &v)) != MLA_OK) return s;
+    if (batch < 0 || q_len < 1 || q_len > 16 || num_splits < 0 || num_splits > 65535) return MLA_ERR_INVALID_ARG;
+    if (max_kv_len < q_len || max_kv_len > cache->capacity) return MLA_ERR_INVALID_ARG;
+    if (batch == 0) return MLA_OK;
+    if (!kv_len || !q_abs || !o_lat || !aligned16(q_abs) || !aligned16(o_lat)) return MLA_ERR_INVALID_ARG;
+    unsigned *status = nullptr;
+    int sms = 0;
+    if ((s = device_info(&status, &sms)) != MLA_OK) return s;
+    // partials for B + S - 1 slots must fit the fixed scratch; an automatic
+    // split count shrinks to fit, an explicit one that does not fit is refused
+    const size_t rows = static_cast<size_t>(q_len) * dims->num_heads;
+    const size_t per_slot = rows * dims->rank;
+    auto need = [&](int S) {
+        const size_t slots = static_cast<size_t>(batch) + S - 1;
+        return slots * per_slot + ((slots * rows + 63) & ~size_t{63});
+    };
+    int S = resolve_splits(dims, batch, q_len, max_kv_len, num_splits, sms);
+    if (need(S) > kNoallocScratchFloats) {
+        if (num_splits > 0) return MLA_ERR_UNSUPPORTED;
+        const int64_t slots_max = static_cast<int64_t>((kNoallocScratchFloats - 64) / (per_slot + rows));
+        S = static_cast<int>(slots_max - batch + 1);
+        while (S >= 1 && need(S) > kNoallocScratchFloats) --S;
+        if (S < 1) return MLA_ERR_UNSUPPORTED;
+    }
+    float *scratch = nullptr;
+    if ((s = noalloc_scratch(&scratch)) != MLA_OK) return s;
+    const size_t slots = static_cast<size_t>(batch) + S - 1;
+    float *o_part = scratch;
+    float *lse_part = scratch + ((slots * per_slot + 63) & ~size_t{63});
+    AttnArgs a;
+    a.batch = batch;
+    a.q_len = q_len;
+    a.num_heads = dims->num_heads;
+    a.rank = dims->rank;
+    a.d_rope = dims->d_rope;
+    a.sm_scale = dims->sm_scale;
+    a.kv_len = kv_len;
+    a.max_kv = max_kv_len;
+    a.q_abs = q_abs;
+    a.num_splits = S;
+    a.o_part = o_part;
+    a.lse_part = lse_part;
+    a.cache = v;
+    a.status = status;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if ((s = from_cuda(use_tc_kernel(dims) ? launch_attn_tc(a, st) : launch_attn_simt(a, st))) != MLA_OK) return s;
+    return from_cuda(launch_combine(batch, q_len, dims->num_heads, dims->rank, max_kv_len, S, kv_len, o_part,
+                                    lse_part, o_lat, lse, st));
 }
 
 const char *mla_last_error(void)
