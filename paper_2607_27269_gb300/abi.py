@@ -58,7 +58,8 @@ def lib(auto_build: bool = True):
     global _lib
     with _lock:
         if _lib is None:
-            path = _build.build() if auto_build else _build.LIB
+            # GBMLA_LIBRARY selects another build of the library (e.g. the trace build)
+            path = os.environ.get("GBMLA_LIBRARY") or (_build.build() if auto_build else _build.LIB)
             if not os.path.exists(path):
                 raise RuntimeError(f"libgbmla.so is missing at {path}; run paper_2607_27269_gb300.build.build()")
             L = ctypes.CDLL(path)

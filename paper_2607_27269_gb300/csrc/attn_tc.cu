@@ -37,6 +37,26 @@ constexpr int kMaxSlots = 16;
 constexpr int kSoftmaxWarps = 12;
 constexpr int kThreads = 64 + 32 * kSoftmaxWarps;
 
+// Optional event trace of the first CTA (compiled only with -DGBMLA_TRACE):
+// (globaltimer ns, event code, argument) triples in a caller buffer, set by
+// mla_debug_trace().  Used to read the per-tile timeline of the roles.
+#ifdef GBMLA_TRACE
+__device__ unsigned long long *g_trace_buf;
+__device__ unsigned g_trace_count;
+__device__ unsigned g_trace_cap;
+__device__ __forceinline__ void trace_event(int code, int64_t arg)
+{
+    if (blockIdx.x != 0 || blockIdx.y != 0 || g_trace_buf == nullptr) return;
+    const unsigned i = atomicAdd(&g_trace_count, 1u);
+    if (i >= g_trace_cap) return;
+    g_trace_buf[2 * i] = global_ns();
+    g_trace_buf[2 * i + 1] = (static_cast<unsigned long long>(code) << 48) | (static_cast<unsigned long long>(arg) & 0xffffffffffffull);
+}
+#define GBMLA_TRACE_EVENT(code, arg) trace_event((code), (arg))
+#else
+#define GBMLA_TRACE_EVENT(code, arg) ((void)0)
+#endif
+
 struct TcArgs {
     int batch, q_len, heads, rank, d_rope, rows, num_splits, max_kv;
     int paged, bt_stride, num_pages, c_slots;
@@ -338,6 +358,7 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
         const int kv = a.kv_len[b];
         const int sb = static_cast<int>(t & 1);
         sm_wait<N>(c, a, ss, &bars.s_full[sb], static_cast<uint32_t>((t >> 1) & 1));
+        if (c.tid == 64) GBMLA_TRACE_EVENT(6, t);
         named_sync_softmax();
         if (ss.sm_fail) break;
         tc::fence_after_sync();
@@ -410,7 +431,9 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
         named_sync_softmax();
         // ---- P is rewritten and O^T rescaled only once PV(t-1) has completed
         if (!first) {
+            if (c.tid == 64) GBMLA_TRACE_EVENT(7, t);
             sm_wait<N>(c, a, ss, &bars.pv_done, static_cast<uint32_t>((t - 1) & 1));
+            if (c.tid == 64) GBMLA_TRACE_EVENT(8, t);
             named_sync_softmax();
             if (ss.sm_fail) break;
             tc::fence_after_sync();
@@ -467,6 +490,7 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
         tc::fence_before_sync();
         __syncwarp();
         if (c.lane == 0) tc::mbar_arrive(smem_u32(&bars.p_full));
+        if (c.tid == 64) GBMLA_TRACE_EVENT(9, t);
         // ---- tail tile: rows past the sequence end in the PV copy of the
         // latent chunks are cleared, so stale or uninitialised bytes never meet
         // a zero weight.  P is already published; the MMA warp reports each
@@ -595,6 +619,7 @@ __global__ void __maxnreg__(128)
                         break;
                     }
                     const uint32_t full = smem_u32(&bars.full[rp.slot]);
+                    GBMLA_TRACE_EVENT(1, chunk_no);
                     tc::mbar_arrive_expect_tx(full, bytes);
                     if (chunk_no % CL == rank_in_cluster) {
                         const uint32_t dst = smem_u32(ring + rp.slot * kChunkBytes);
@@ -695,6 +720,7 @@ __global__ void __maxnreg__(128)
                     if (!wait(&bars.q_full, seg_q & 1)) return;
                 }
                 const int sb = tq & 1;
+                GBMLA_TRACE_EVENT(2, tq);
                 if (tq >= 2 && !wait(&bars.s_free[sb], ((tq >> 1) - 1) & 1)) return;
                 if (!wait(&bars.kr_full, kr_uses & 1)) return;
                 tc::fence_after_sync();
@@ -717,12 +743,14 @@ __global__ void __maxnreg__(128)
                     rp.advance(CS);
                 }
                 tc::commit(smem_u32(&bars.s_full[sb]));
+                GBMLA_TRACE_EVENT(3, tq);
                 if (wq.last()) tc::commit(smem_u32(&bars.q_free));
                 ++tq;
                 wq.next();
             };
             auto do_pv = [&](int t) {
                 if (!wait(&bars.p_full, t & 1)) return;
+                GBMLA_TRACE_EVENT(4, t);
                 bool first_pv = false;
                 if (wp.first()) {
                     ++seg_p;
@@ -753,6 +781,7 @@ __global__ void __maxnreg__(128)
                     rp.advance(CS);
                 }
                 tc::commit(smem_u32(&bars.pv_done));
+                GBMLA_TRACE_EVENT(5, t);
                 if (tail) ++n_tail;
                 wp.next();
             };
@@ -972,3 +1001,16 @@ cudaError_t launch_attn_tc(const AttnArgs &a, cudaStream_t st)
 }
 
 }  // namespace gbmla
+
+#ifdef GBMLA_TRACE
+// Trace builds only: record the first CTA's events into `buf` (2 x 64-bit
+// words per event, at most `cap` events).  Returns the CUDA status.
+extern "C" int mla_debug_trace(unsigned long long *buf, unsigned cap)
+{
+    const unsigned zero = 0;
+    if (cudaMemcpyToSymbol(gbmla::g_trace_buf, &buf, sizeof buf) != cudaSuccess) return 1;
+    if (cudaMemcpyToSymbol(gbmla::g_trace_cap, &cap, sizeof cap) != cudaSuccess) return 1;
+    if (cudaMemcpyToSymbol(gbmla::g_trace_count, &zero, sizeof zero) != cudaSuccess) return 1;
+    return 0;
+}
+#endif
