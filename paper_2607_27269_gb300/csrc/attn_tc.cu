@@ -6,19 +6,20 @@
 //     S^T [128 tok, N] = [k_rope | c] tile (K-major A) x q_abs^T (K-major B)
 //     online softmax over tokens (TMEM lane = token, column = query row)
 //     O^T [r, N]      += C^T (latent tile read as an MN-major A) x P^T
-// S^T (two buffers) and O^T live in TMEM.  The latent tile streams through a
-// ring of 64-column chunks twice, once for each product, in the order the MMA
-// warp consumes them: QK(0), QK(1), PV(0), QK(2), PV(1), ... so that the
-// softmax of tile t overlaps QK(t+1).  The second pass reads from L2.  The
-// positional keys use a buffer of their own.  With two query groups (160 query
-// rows) the two CTAs form a cluster and every cache box is multicast to both,
-// so each byte leaves L2 once per pass.
+// S^T (two buffers) and O^T live in TMEM.  The cache streams through two
+// rings of 64-column chunks: the QK ring (positional keys, then the latent
+// chunks of each tile) feeds the score products, the PV ring (the latent
+// chunks again, from L2) the value products, so that the softmax of tile t
+// overlaps QK(t+1) and PV(t-1).  With two query groups (160 query rows) the
+// two CTAs form a cluster and every cache box is multicast to both, so each
+// byte leaves L2 once per pass.
 //
-// Warp roles (448 threads): warp 0 = TMA producer, warp 1 = MMA issuer and
-// TMEM owner, warps 2..13 = softmax / epilogue (three warps per TMEM lane
-// quarter, each owning every third 16-column block of the query columns).  Every wait is bounded; a
-// wait that runs out records a timeout in the status word and the CTA winds
-// down without trapping.
+// Warp roles (512 threads): warps 0 and 3 = TMA producers (QK ring and query
+// boxes; PV ring), warp 1 = QK MMA issuer and TMEM owner, warp 2 = PV MMA
+// issuer, warps 4..15 = softmax / epilogue (three warps per TMEM lane quarter,
+// each owning every third 16-column block of the query columns).  Every wait
+// is bounded; a wait that runs out records a timeout in the status word and
+// the CTA winds down without trapping.
 #include <cudaTypedefs.h>
 #include <math.h>
 #include <stdlib.h>
@@ -33,9 +34,10 @@ namespace {
 constexpr int kTile = MLA_SPLIT_TILE;     // tokens per tile (MMA M)
 constexpr int kHalf = 64;                 // tokens per TMA box (one page when paged)
 constexpr int kChunkBytes = kTile * 128;  // 128 tokens x 64 bf16 columns, SW128 K-major
-constexpr int kMaxSlots = 16;
+constexpr int kMaxSlots = 16;               // ring slots of both rings together
 constexpr int kSoftmaxWarps = 12;
-constexpr int kThreads = 64 + 32 * kSoftmaxWarps;
+constexpr int kSoftmaxBase = 128;           // first softmax thread (after two producer and two MMA warps)
+constexpr int kThreads = kSoftmaxBase + 32 * kSoftmaxWarps;
 
 // Optional event trace of the first CTA (compiled only with -DGBMLA_TRACE):
 // (globaltimer ns, event code, argument) triples in a caller buffer, set by
@@ -44,10 +46,11 @@ constexpr int kThreads = 64 + 32 * kSoftmaxWarps;
 __device__ unsigned long long *g_trace_buf;
 __device__ unsigned g_trace_count;
 __device__ unsigned g_trace_cap;
+__shared__ unsigned s_trace_count;  // events of this CTA (a shared-memory atomic keeps the probe cheap)
 __device__ __forceinline__ void trace_event(int code, int64_t arg)
 {
     if (blockIdx.x != 0 || blockIdx.y != 0 || g_trace_buf == nullptr) return;
-    const unsigned i = atomicAdd(&g_trace_count, 1u);
+    const unsigned i = atomicAdd(&s_trace_count, 1u);
     if (i >= g_trace_cap) return;
     g_trace_buf[2 * i] = global_ns();
     g_trace_buf[2 * i + 1] = (static_cast<unsigned long long>(code) << 48) | (static_cast<unsigned long long>(arg) & 0xffffffffffffull);
@@ -59,7 +62,7 @@ __device__ __forceinline__ void trace_event(int code, int64_t arg)
 
 struct TcArgs {
     int batch, q_len, heads, rank, d_rope, rows, num_splits, max_kv;
-    int paged, bt_stride, num_pages, c_slots;
+    int paged, bt_stride, num_pages, qk_slots, pv_slots;
     float scale_log2;
     const int32_t *kv_len;
     const int32_t *block_table;
@@ -69,13 +72,14 @@ struct TcArgs {
 };
 
 struct __align__(8) Bars {
-    uint64_t full[kMaxSlots], empty[kMaxSlots];
-    uint64_t kr_full, kr_empty, q_full, q_free;
+    uint64_t qk_full[kMaxSlots], qk_empty[kMaxSlots];  // QK ring: positional keys + latent chunks
+    uint64_t pv_full[kMaxSlots], pv_empty[kMaxSlots];  // PV ring: latent chunks again
+    uint64_t q_full, q_free;
     uint64_t s_full[2], s_free[2];
-    uint64_t p_full, pv_done, o_free, drain;
-    // Tail tile handshake per r-chunk m: the MMA warp (which waits on `full`
-    // in strict order) reports that chunks 2m, 2m+1 of the PV copy landed
-    // (zready); the softmax warps clear their rows past the end (zdone).
+    uint64_t p_full, pv_done, o_free, drain_qk, drain_pv;
+    // Tail tile handshake per r-chunk m: the PV warp (which waits on its
+    // ring in strict order) reports that chunks 2m, 2m+1 landed (zready);
+    // the softmax warps clear their rows past the end (zdone).
     uint64_t zready[4], zdone[4];
 };
 
@@ -134,32 +138,37 @@ struct Walk {
     }
 };
 
-// Where the (up to) two 64-token halves of tile j of sequence b live.
+// Where the boxes of tile j of sequence b live: a contiguous cache loads
+// the tile as one 128-row box, a paged cache as one 64-row box per page.
 struct TileLoc {
-    int nh;            // halves to load (1 or 2; 0 if the first page is bad)
+    int nh;            // boxes to load (0 if the first page is bad)
+    uint32_t bytes;    // bytes the boxes deliver
     int32_t tok0[2], blk[2];
 };
 
 __device__ __forceinline__ TileLoc locate(const TcArgs &a, int b, int j)
 {
     TileLoc L;
+    if (!a.paged) {
+        L.nh = 1;
+        L.bytes = kTile * 128;
+        L.blk[0] = b;
+        L.tok0[0] = j * kTile;
+        return L;
+    }
     const int kv = a.kv_len[b];
     L.nh = (kv - j * kTile > kHalf) ? 2 : 1;
     for (int h = 0; h < L.nh; ++h) {
-        if (a.paged) {
-            const int32_t pg = a.block_table[static_cast<int64_t>(b) * a.bt_stride + 2 * j + h];
-            if (pg < 0 || pg >= a.num_pages) {
-                record_status(a.status, kStatusBounds);
-                L.nh = h;
-                break;
-            }
-            L.blk[h] = pg;
-            L.tok0[h] = 0;
-        } else {
-            L.blk[h] = b;
-            L.tok0[h] = j * kTile + h * kHalf;
+        const int32_t pg = a.block_table[static_cast<int64_t>(b) * a.bt_stride + 2 * j + h];
+        if (pg < 0 || pg >= a.num_pages) {
+            record_status(a.status, kStatusBounds);
+            L.nh = h;
+            break;
         }
+        L.blk[h] = pg;
+        L.tok0[h] = 0;
     }
+    L.bytes = static_cast<uint32_t>(L.nh) * kHalf * 128;
     return L;
 }
 
@@ -174,6 +183,18 @@ struct RingPos {
         }
     }
 };
+
+// Non-blocking test: has the phase with this parity completed?
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
 
 __device__ __forceinline__ void named_sync_softmax()
 {
@@ -237,13 +258,13 @@ struct SmCtx {
     int64_t t_begin, t_end;
 };
 
-// One lane of the warp waits; a failure marks sm_fail, which the softmax
+// The whole warp waits; a failure marks sm_fail, which the softmax
 // warps read only after their next named barrier, so they all leave together.
 template <int N>
 __device__ __forceinline__ void sm_wait(const SmCtx &c, const TcArgs &a, Shared<N> &ss, uint64_t *bar,
                                         uint32_t parity)
 {
-    if (c.lane == 0 && !mbar_wait(smem_u32(bar), parity, c.lim_ns)) {
+    if (!__all_sync(0xffffffffu, mbar_wait(smem_u32(bar), parity, c.lim_ns)) && c.lane == 0) {
         record_status(a.status, kStatusTimeout);
         atomicOr(&ss.sm_fail, 1);
         ss.abort = 1;
@@ -303,7 +324,7 @@ __device__ __forceinline__ void sm_epilogue(const SmCtx &c, const TcArgs &a, Sha
         }
     }
     named_sync_softmax();
-    const int cc = c.tid - 64;
+    const int cc = c.tid - kSoftmaxBase;
     if (cc < N) {
         const float l = ss.red[0][cc] + ss.red[1][cc] + ss.red[2][cc] + ss.red[3][cc];
         ss.lsum[cc] = l;
@@ -349,7 +370,7 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
     int b_cur = -1;
     int64_t t_last = -1;
     int n_tail = 0;  // tail tiles handled so far (phase of zready / zdone)
-    const int cc = c.tid - 64;
+    const int cc = c.tid - kSoftmaxBase;
     Walk w;
     w.init(a.kv_len, a.batch, a.q_len, a.max_kv, c.t_begin, c.t_end);
     for (int64_t t = 0; !w.done(); ++t, w.next()) {
@@ -358,7 +379,7 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
         const int kv = a.kv_len[b];
         const int sb = static_cast<int>(t & 1);
         sm_wait<N>(c, a, ss, &bars.s_full[sb], static_cast<uint32_t>((t >> 1) & 1));
-        if (c.tid == 64) GBMLA_TRACE_EVENT(6, t);
+        if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(6, t);
         named_sync_softmax();
         if (ss.sm_fail) break;
         tc::fence_after_sync();
@@ -392,7 +413,7 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
                 ss.m_used[cc] = fmaxf(fmaxf(ss.red[0][cc], ss.red[1][cc]), fmaxf(ss.red[2][cc], ss.red[3][cc]));
                 ss.alpha[cc] = 1.f;
             }
-            if (c.tid == 64) ss.any_rescale = 0;
+            if (c.tid == kSoftmaxBase) ss.any_rescale = 0;
         } else {
             bool over = false;
 #pragma unroll
@@ -420,20 +441,20 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
                     }
                     ss.alpha[cc] = alpha;
                 }
-                if (c.tid == 64) {
+                if (c.tid == kSoftmaxBase) {
                     ss.any_rescale = 1;
                     ss.need_max = 0;
                 }
-            } else if (c.tid == 64) {
+            } else if (c.tid == kSoftmaxBase) {
                 ss.any_rescale = 0;
             }
         }
         named_sync_softmax();
         // ---- P is rewritten and O^T rescaled only once PV(t-1) has completed
         if (!first) {
-            if (c.tid == 64) GBMLA_TRACE_EVENT(7, t);
+            if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(7, t);
             sm_wait<N>(c, a, ss, &bars.pv_done, static_cast<uint32_t>((t - 1) & 1));
-            if (c.tid == 64) GBMLA_TRACE_EVENT(8, t);
+            if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(8, t);
             named_sync_softmax();
             if (ss.sm_fail) break;
             tc::fence_after_sync();
@@ -490,15 +511,14 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
         tc::fence_before_sync();
         __syncwarp();
         if (c.lane == 0) tc::mbar_arrive(smem_u32(&bars.p_full));
-        if (c.tid == 64) GBMLA_TRACE_EVENT(9, t);
+        if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(9, t);
         // ---- tail tile: rows past the sequence end in the PV copy of the
         // latent chunks are cleared, so stale or uninitialised bytes never meet
         // a zero weight.  P is already published; the MMA warp reports each
         // landed pair (zready) and waits for it to be cleared (zdone), so every
         // wait here is on the next phase of its barrier.
         if (last && kv - j * kTile < kTile) {
-            const int64_t qk_groups = (t + 2 < c.n_items) ? t + 2 : c.n_items;
-            const int64_t g0 = static_cast<int64_t>(c.ncc) * (qk_groups + t);
+            const int64_t g0 = static_cast<int64_t>(c.ncc) * t;  // first PV-ring chunk of tile t
             for (int m = 0; m < c.nrc; ++m) {
                 sm_wait<N>(c, a, ss, &bars.zready[m], static_cast<uint32_t>(n_tail & 1));
                 if (pos >= kv) {
@@ -526,7 +546,6 @@ __global__ void __maxnreg__(128)
     attn_tc_kernel(const __grid_constant__ TcArgs a, const __grid_constant__ CUtensorMap map_c,
                    const __grid_constant__ CUtensorMap map_r, const __grid_constant__ CUtensorMap map_q)
 {
-    constexpr int NB = N / 16;                   // 16-column blocks
     constexpr uint16_t kMask = (1u << CL) - 1;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     __shared__ Bars bars;
@@ -537,11 +556,13 @@ __global__ void __maxnreg__(128)
                                                             ~static_cast<uintptr_t>(1023));
     const int ncc = a.rank / 64;    // latent chunks per tile
     const int nrc = a.rank / 128;   // r-chunks of O^T
-    const int CS = a.c_slots;       // ring slots (even)
-    unsigned char *q_buf = smem;                                                // (ncc+1) x [N x 128 B]
-    unsigned char *kr_buf = q_buf + (((ncc + 1) * N * 128 + 1023) & ~1023);     // [128 x 128 B]
-    unsigned char *ring = kr_buf + kChunkBytes;                                 // CS x [128 x 128 B]
-    unsigned char *p_buf = ring + CS * kChunkBytes;                             // NB x [128 tok x 32 B]
+    const int nqc = ncc + 1;        // chunks of a tile in the QK pass: positional keys, then latent
+    const int CA = a.qk_slots;      // QK ring slots
+    const int CB = a.pv_slots;      // PV ring slots (even)
+    unsigned char *q_buf = smem;                                          // nqc x [N x 128 B]
+    unsigned char *ring_a = q_buf + ((nqc * N * 128 + 1023) & ~1023);     // CA x [128 x 128 B]
+    unsigned char *ring_b = ring_a + CA * kChunkBytes;                    // CB x [128 x 128 B]
+    unsigned char *p_buf = ring_b + CB * kChunkBytes;                     // NB x [128 tok x 32 B]
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int group = blockIdx.x, part = blockIdx.y;
@@ -561,11 +582,11 @@ __global__ void __maxnreg__(128)
 
     if (tid == 0) {
         for (int i = 0; i < kMaxSlots; ++i) {
-            mbar_init(&bars.full[i], 1);
-            mbar_init(&bars.empty[i], CL);
+            mbar_init(&bars.qk_full[i], 1);
+            mbar_init(&bars.qk_empty[i], CL);
+            mbar_init(&bars.pv_full[i], 1);
+            mbar_init(&bars.pv_empty[i], CL);
         }
-        mbar_init(&bars.kr_full, 1);
-        mbar_init(&bars.kr_empty, CL);
         mbar_init(&bars.q_full, 1);
         mbar_init(&bars.q_free, 1);
         for (int i = 0; i < 2; ++i) {
@@ -575,11 +596,15 @@ __global__ void __maxnreg__(128)
         mbar_init(&bars.p_full, kSoftmaxWarps);
         mbar_init(&bars.pv_done, 1);
         mbar_init(&bars.o_free, kSoftmaxWarps);
-        mbar_init(&bars.drain, 1);
+        mbar_init(&bars.drain_qk, 1);
+        mbar_init(&bars.drain_pv, 1);
         for (int i = 0; i < 4; ++i) {
             mbar_init(&bars.zready[i], 1);
             mbar_init(&bars.zdone[i], kSoftmaxWarps);
         }
+#ifdef GBMLA_TRACE
+        s_trace_count = 0;
+#endif
         ss.need_max = 0;
         ss.any_rescale = 0;
         ss.abort = 0;
@@ -597,99 +622,124 @@ __global__ void __maxnreg__(128)
     tc::fence_after_sync();
     const uint32_t tmem = ss.tmem_base;
     const uint32_t o_col0 = 2 * N;   // S^T buffers at columns [0, N) and [N, 2N)
+    auto any_abort = [&]() {
+        return __any_sync(0xffffffffu, *reinterpret_cast<volatile int *>(&ss.abort) != 0);
+    };
 
-    if (warp == 0) {
-        // ================================================================ TMA producer
-        if (lane == 0 && n_items > 0) {
-            tc::prefetch_tensormap(&map_c);
-            tc::prefetch_tensormap(&map_r);
-            tc::prefetch_tensormap(&map_q);
-            Walk wq, wp;
-            wq.init(a.kv_len, a.batch, a.q_len, a.max_kv, t_begin, t_end);
-            wp.init(a.kv_len, a.batch, a.q_len, a.max_kv, t_begin, t_end);
-            RingPos rp{0, 0};
-            int kr_uses = 0, seg = -1;
-            int64_t chunk_no = 0;
+    if (warp == 0 || warp == 3) {
+        // ================================================================ TMA producers
+        // A tensor-TMA instruction occupies its issuing thread for a long,
+        // nearly size-independent time, so the loads are spread over lanes
+        // and warps, each lane an independent in-order stream.  Warp 0: lane
+        // s < CA refills QK-ring slot s (chunks s, s + CA, ... of the QK pass,
+        // nqc per tile: positional keys, then the latent chunks), lanes
+        // 16..16+ncc load the query boxes of each sequence.  Warp 3: lane s <
+        // CB refills PV-ring slot s (chunks s, s + CB, ... of the PV pass, ncc
+        // per tile).  The lanes of a warp poll their own barrier without
+        // blocking in one converged loop, and every lane whose slot is free
+        // issues in the same pass.  A lane waits only on phases of its own
+        // barrier, in order, so every parity test is on the next phase.
+        if (n_items > 0) {
+            if (lane == 0 && warp == 0) {
+                tc::prefetch_tensormap(&map_c);
+                tc::prefetch_tensormap(&map_r);
+                tc::prefetch_tensormap(&map_q);
+            }
+            enum { kQK, kPV, kQuery, kIdle };
+            const int kind = warp == 3 ? (lane < CB ? kPV : kIdle)
+                                       : (lane < CA ? kQK : (lane >= 16 && lane < 16 + nqc) ? kQuery : kIdle);
+            const int slot = lane;
+            const int per_tile = kind == kQK ? nqc : ncc;
+            const int ring_len = kind == kQK ? CA : CB;
+            Walk w;
+            w.init(a.kv_len, a.batch, a.q_len, a.max_kv, t_begin, t_end);
+            const int64_t total = static_cast<int64_t>(n_items) * per_tile;
+            int64_t c = slot;  // ring lanes: next chunk of this lane's pass
+            int64_t k = 0;     // jobs this lane has issued (ring round / sequence)
+            bool has = (kind == kQK || kind == kPV) ? c < total : kind == kQuery;
             bool ok = true;
-            auto load_chunks = [&](const TileLoc &L) {
-                const uint32_t bytes = static_cast<uint32_t>(L.nh) * kHalf * 128;
-                for (int i = 0; i < ncc && ok; ++i) {
-                    if (rp.round >= 1 && !mbar_wait(smem_u32(&bars.empty[rp.slot]), (rp.round - 1) & 1, lim_ns)) {
-                        ok = false;
-                        break;
-                    }
-                    const uint32_t full = smem_u32(&bars.full[rp.slot]);
-                    GBMLA_TRACE_EVENT(1, chunk_no);
-                    tc::mbar_arrive_expect_tx(full, bytes);
-                    if (chunk_no % CL == rank_in_cluster) {
-                        const uint32_t dst = smem_u32(ring + rp.slot * kChunkBytes);
-                        for (int h = 0; h < L.nh; ++h) {
-                            if (CL > 1)
-                                tc::tma_load_3d_multicast(dst + h * kHalf * 128, &map_c, 64 * i, L.tok0[h], L.blk[h],
-                                                          full, kMask);
-                            else
-                                tc::tma_load_3d(dst + h * kHalf * 128, &map_c, 64 * i, L.tok0[h], L.blk[h], full);
+            uint64_t wait_t0 = 0;
+            uint32_t wbar = 0, fbar = 0, dst = 0;
+            if (kind == kQK) {
+                wbar = smem_u32(&bars.qk_empty[slot]);
+                fbar = smem_u32(&bars.qk_full[slot]);
+                dst = smem_u32(ring_a + slot * kChunkBytes);
+            } else if (kind == kPV) {
+                wbar = smem_u32(&bars.pv_empty[slot]);
+                fbar = smem_u32(&bars.pv_full[slot]);
+                dst = smem_u32(ring_b + slot * kChunkBytes);
+            } else if (kind == kQuery) {
+                wbar = smem_u32(&bars.q_free);
+                fbar = smem_u32(&bars.q_full);
+                dst = smem_u32(q_buf + (lane - 16) * N * 128);
+            }
+            while (true) {
+                if (kind == kQuery) has = has && !w.done();
+                if (!__any_sync(0xffffffffu, has && ok)) break;
+                if (any_abort()) break;
+                bool progressed = false;
+                if (has && ok) {
+                    const bool ready = k == 0 || mbar_test(wbar, static_cast<uint32_t>((k - 1) & 1));
+                    if (!ready) {
+                        const uint64_t now = global_ns();
+                        if (wait_t0 == 0)
+                            wait_t0 = now;
+                        else if (now - wait_t0 > lim_ns)
+                            ok = false;
+                    } else {
+                        wait_t0 = 0;
+                        progressed = true;
+                        if (kind == kQuery) {
+                            const int box = lane - 16;
+                            if (box == 0) tc::mbar_arrive_expect_tx(fbar, nqc * N * 128);
+                            tc::tma_load_2d(dst, &map_q, 64 * box, w.b * a.rows + group * N, fbar);
+                            do {
+                                w.next();
+                            } while (!w.done() && !w.first());
+                        } else {
+                            const int64_t tile = c / per_tile;
+                            const int i = static_cast<int>(c - tile * per_tile);
+                            while (w.t < t_begin + tile) w.next();
+                            const TileLoc L = locate(a, w.b, w.tile());
+                            // QK pass: chunk 0 = positional keys, 1.. = latent; PV pass: latent
+                            const bool keys = kind == kQK && i == 0;
+                            const CUtensorMap *map = keys ? &map_r : &map_c;
+                            const int col = keys ? 0 : 64 * (kind == kQK ? i - 1 : i);
+                            if (lane == 0 && warp == 0) GBMLA_TRACE_EVENT(1, c);
+                            tc::mbar_arrive_expect_tx(fbar, L.bytes);
+                            if (c % CL == rank_in_cluster) {
+                                for (int h = 0; h < L.nh; ++h) {
+                                    if (CL > 1)
+                                        tc::tma_load_3d_multicast(dst + h * kHalf * 128, map, col, L.tok0[h],
+                                                                  L.blk[h], fbar, kMask);
+                                    else
+                                        tc::tma_load_3d(dst + h * kHalf * 128, map, col, L.tok0[h], L.blk[h], fbar);
+                                }
+                            }
+                            c += ring_len;
+                            has = c < total;
                         }
-                    }
-                    ++chunk_no;
-                    rp.advance(CS);
-                }
-            };
-            auto emit_qk = [&]() {
-                const int b = wq.b, j = wq.tile();
-                if (wq.first()) {
-                    ++seg;
-                    if (seg >= 1 && !mbar_wait(smem_u32(&bars.q_free), (seg - 1) & 1, lim_ns)) {
-                        ok = false;
-                        return;
-                    }
-                    tc::mbar_arrive_expect_tx(smem_u32(&bars.q_full), (ncc + 1) * N * 128);
-                    for (int i = 0; i <= ncc; ++i)
-                        tc::tma_load_2d(smem_u32(q_buf + i * N * 128), &map_q, 64 * i, b * a.rows + group * N,
-                                        smem_u32(&bars.q_full));
-                }
-                const TileLoc L = locate(a, b, j);
-                if (kr_uses >= 1 && !mbar_wait(smem_u32(&bars.kr_empty), (kr_uses - 1) & 1, lim_ns)) {
-                    ok = false;
-                    return;
-                }
-                const uint32_t krf = smem_u32(&bars.kr_full);
-                tc::mbar_arrive_expect_tx(krf, static_cast<uint32_t>(L.nh) * kHalf * 128);
-                if (kr_uses % CL == static_cast<int>(rank_in_cluster)) {
-                    for (int h = 0; h < L.nh; ++h) {
-                        if (CL > 1)
-                            tc::tma_load_3d_multicast(smem_u32(kr_buf) + h * kHalf * 128, &map_r, 0, L.tok0[h],
-                                                      L.blk[h], krf, kMask);
-                        else
-                            tc::tma_load_3d(smem_u32(kr_buf) + h * kHalf * 128, &map_r, 0, L.tok0[h], L.blk[h], krf);
+                        ++k;
                     }
                 }
-                ++kr_uses;
-                load_chunks(L);
-                wq.next();
-            };
-            auto emit_pv = [&]() {
-                load_chunks(locate(a, wp.b, wp.tile()));
-                wp.next();
-            };
-            emit_qk();
-            for (int t = 0; t < n_items && ok && !*reinterpret_cast<volatile int *>(&ss.abort); ++t) {
-                if (t + 1 < n_items) emit_qk();
-                if (!ok) break;
-                emit_pv();
+                if (!__any_sync(0xffffffffu, progressed)) __nanosleep(32);
             }
             if (!ok) {
                 record_status(a.status, kStatusTimeout);
                 ss.abort = 1;
             }
+            __syncwarp();
         }
-    } else if (warp == 1) {
-        // ================================================================ MMA issuer
-        if (lane == 0 && n_items > 0) {
-            const uint32_t id_qk = tc::idesc_bf16_f32(128, N, false, false);
-            const uint32_t id_pv = tc::idesc_bf16_f32(128, N, true, true);
-            const uint32_t q_base = smem_u32(q_buf), kr_base = smem_u32(kr_buf);
-            const uint32_t ring_base = smem_u32(ring), p_base = smem_u32(p_buf);
+    } else if (warp == 1 || warp == 2) {
+        // ================================================================ MMA issuers
+        // Warp 1 issues the score products QK(t), warp 2 the value products
+        // PV(t); each consumes its own ring in order.  The whole warp runs its
+        // loop converged (every lane waits); one elected lane issues each MMA,
+        // commit and arrive.
+        const bool is_qk = warp == 1;
+        uint64_t *drain = is_qk ? &bars.drain_qk : &bars.drain_pv;
+        if (n_items > 0) {
+            const uint32_t q_base = smem_u32(q_buf), p_base = smem_u32(p_buf);
             // descriptor templates (start address added per MMA)
             const uint64_t dq = tc::smem_desc(0, 16, 1024, tc::kSwizzle128B);
             const uint64_t dc = tc::smem_desc(0, kChunkBytes, 1024, tc::kSwizzle128B);
@@ -697,107 +747,108 @@ __global__ void __maxnreg__(128)
             auto with_addr = [](uint64_t tmpl, uint32_t saddr) {
                 return tmpl | static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
             };
-            Walk wq, wp;
-            wq.init(a.kv_len, a.batch, a.q_len, a.max_kv, t_begin, t_end);
-            wp.init(a.kv_len, a.batch, a.q_len, a.max_kv, t_begin, t_end);
+            Walk w;
+            w.init(a.kv_len, a.batch, a.q_len, a.max_kv, t_begin, t_end);
             RingPos rp{0, 0};
-            int kr_uses = 0, seg_q = -1, seg_p = -1, tq = 0, n_tail = 0;
             bool ok = true;
             auto wait = [&](uint64_t *bar, uint32_t parity) {
-                if (ok && !mbar_wait(smem_u32(bar), parity, lim_ns)) ok = false;
+                if (ok) ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(bar), parity, lim_ns));
                 return ok;
             };
             // a consumed slot is handed back to every CTA of the cluster
             auto release = [&](uint64_t *bar) {
                 if (CL > 1)
-                    tc::commit_multicast(smem_u32(bar), kMask);
+                    tc::commit_multicast_elect(smem_u32(bar), kMask);
                 else
-                    tc::commit(smem_u32(bar));
+                    tc::commit_elect(smem_u32(bar));
             };
-            auto do_qk = [&]() {
-                if (wq.first()) {
-                    ++seg_q;
-                    if (!wait(&bars.q_full, seg_q & 1)) return;
-                }
-                const int sb = tq & 1;
-                GBMLA_TRACE_EVENT(2, tq);
-                if (tq >= 2 && !wait(&bars.s_free[sb], ((tq >> 1) - 1) & 1)) return;
-                if (!wait(&bars.kr_full, kr_uses & 1)) return;
-                tc::fence_after_sync();
-                const uint32_t d_s = tmem + sb * N;
-                const uint32_t qr = q_base + ncc * N * 128;
-#pragma unroll
-                for (int k = 0; k < 4; ++k)
-                    tc::mma_bf16(d_s, with_addr(dq, kr_base + k * 32), with_addr(dq, qr + k * 32), id_qk, k > 0);
-                release(&bars.kr_empty);
-                ++kr_uses;
-                for (int i = 0; i < ncc; ++i) {
-                    if (!wait(&bars.full[rp.slot], rp.round & 1)) return;
-                    tc::fence_after_sync();
-                    const uint32_t cb = ring_base + rp.slot * kChunkBytes;
-                    const uint32_t qb = q_base + i * N * 128;
-#pragma unroll
-                    for (int k = 0; k < 4; ++k)
-                        tc::mma_bf16(d_s, with_addr(dq, cb + k * 32), with_addr(dq, qb + k * 32), id_qk, 1);
-                    release(&bars.empty[rp.slot]);
-                    rp.advance(CS);
-                }
-                tc::commit(smem_u32(&bars.s_full[sb]));
-                GBMLA_TRACE_EVENT(3, tq);
-                if (wq.last()) tc::commit(smem_u32(&bars.q_free));
-                ++tq;
-                wq.next();
-            };
-            auto do_pv = [&](int t) {
-                if (!wait(&bars.p_full, t & 1)) return;
-                GBMLA_TRACE_EVENT(4, t);
-                bool first_pv = false;
-                if (wp.first()) {
-                    ++seg_p;
-                    if (seg_p >= 1 && !wait(&bars.o_free, (seg_p - 1) & 1)) return;
-                    first_pv = true;
-                }
-                // a sequence's last, partial tile: its rows past the end are cleared
-                // by the softmax warps, pair by pair, before PV reads them
-                const bool tail = wp.last() && a.kv_len[wp.b] - wp.tile() * kTile < kTile;
-                for (int m = 0; m < nrc; ++m) {
-                    // chunks 2m, 2m+1 sit in adjacent slots (every group starts at an even slot)
-                    const int s0 = rp.slot;
-                    if (!wait(&bars.full[s0], rp.round & 1) || !wait(&bars.full[s0 + 1], rp.round & 1)) return;
-                    if (tail) {
-                        tc::mbar_arrive(smem_u32(&bars.zready[m]));
-                        if (!wait(&bars.zdone[m], n_tail & 1)) return;
+            if (is_qk) {
+                const uint32_t id_qk = tc::idesc_bf16_f32(128, N, false, false);
+                const uint32_t ring_base = smem_u32(ring_a);
+                int seg = -1;
+                for (int t = 0; t < n_items && ok; ++t, w.next()) {
+                    if (any_abort()) break;
+                    if (w.first()) {
+                        ++seg;
+                        if (!wait(&bars.q_full, seg & 1)) break;
                     }
-                    tc::fence_after_sync();
-                    const uint32_t cb = ring_base + s0 * kChunkBytes;
-                    const uint32_t d_o = tmem + o_col0 + m * N;
+                    const int sb = t & 1;
+                    if (lane == 0) GBMLA_TRACE_EVENT(2, t);
+                    if (t >= 2 && !wait(&bars.s_free[sb], ((t >> 1) - 1) & 1)) break;
+                    const uint32_t d_s = tmem + sb * N;
+                    for (int i = 0; i < nqc && ok; ++i) {
+#ifdef GBMLA_TRACE
+                        if (lane == 0 && !mbar_test(smem_u32(&bars.qk_full[rp.slot]), rp.round & 1))
+                            GBMLA_TRACE_EVENT(12, static_cast<int64_t>(rp.round) * CA + rp.slot);
+#endif
+                        if (!wait(&bars.qk_full[rp.slot], rp.round & 1)) break;
+                        tc::fence_after_sync();
+                        const uint32_t cb = ring_base + rp.slot * kChunkBytes;
+                        const uint32_t qb = q_base + (i == 0 ? ncc : i - 1) * N * 128;
 #pragma unroll
-                    for (int kk = 0; kk < kTile / 16; ++kk)
-                        tc::mma_bf16(d_o, with_addr(dc, cb + kk * 16 * 128), with_addr(dp, p_base + kk * 16 * 32), id_pv,
-                                     (first_pv && kk == 0) ? 0u : 1u);
-                    release(&bars.empty[s0]);
-                    release(&bars.empty[s0 + 1]);
-                    rp.advance(CS);
-                    rp.advance(CS);
+                        for (int kk = 0; kk < 4; ++kk)
+                            tc::mma_bf16_elect(d_s, with_addr(dq, cb + kk * 32), with_addr(dq, qb + kk * 32), id_qk,
+                                               (i | kk) != 0);
+                        release(&bars.qk_empty[rp.slot]);
+                        rp.advance(CA);
+                    }
+                    if (!ok) break;
+                    tc::commit_elect(smem_u32(&bars.s_full[sb]));
+                    if (lane == 0) GBMLA_TRACE_EVENT(3, t);
+                    if (w.last()) tc::commit_elect(smem_u32(&bars.q_free));
                 }
-                tc::commit(smem_u32(&bars.pv_done));
-                GBMLA_TRACE_EVENT(5, t);
-                if (tail) ++n_tail;
-                wp.next();
-            };
-            do_qk();
-            for (int t = 0; t < n_items && ok && !*reinterpret_cast<volatile int *>(&ss.abort); ++t) {
-                if (t + 1 < n_items) do_qk();
-                if (!ok) break;
-                do_pv(t);
+            } else {
+                const uint32_t id_pv = tc::idesc_bf16_f32(128, N, true, true);
+                const uint32_t ring_base = smem_u32(ring_b);
+                int seg = -1, n_tail = 0;
+                for (int t = 0; t < n_items && ok; ++t, w.next()) {
+                    if (any_abort()) break;
+                    if (!wait(&bars.p_full, t & 1)) break;
+                    if (lane == 0) GBMLA_TRACE_EVENT(4, t);
+                    bool first_pv = false;
+                    if (w.first()) {
+                        ++seg;
+                        if (seg >= 1 && !wait(&bars.o_free, (seg - 1) & 1)) break;
+                        first_pv = true;
+                    }
+                    // a sequence's last, partial tile: its rows past the end are cleared
+                    // by the softmax warps, pair by pair, before PV reads them
+                    const bool tail = w.last() && a.kv_len[w.b] - w.tile() * kTile < kTile;
+                    for (int m = 0; m < nrc && ok; ++m) {
+                        // chunks 2m, 2m+1 sit in adjacent slots (CB and ncc are even)
+                        const int s0 = rp.slot;
+                        if (!wait(&bars.pv_full[s0], rp.round & 1) || !wait(&bars.pv_full[s0 + 1], rp.round & 1)) break;
+                        if (tail) {
+                            tc::mbar_arrive_elect(smem_u32(&bars.zready[m]));
+                            if (!wait(&bars.zdone[m], n_tail & 1)) break;
+                        }
+                        tc::fence_after_sync();
+                        const uint32_t cb = ring_base + s0 * kChunkBytes;
+                        const uint32_t d_o = tmem + o_col0 + m * N;
+#pragma unroll
+                        for (int kk = 0; kk < kTile / 16; ++kk)
+                            tc::mma_bf16_elect(d_o, with_addr(dc, cb + kk * 16 * 128),
+                                               with_addr(dp, p_base + kk * 16 * 32), id_pv,
+                                               (first_pv && kk == 0) ? 0u : 1u);
+                        release(&bars.pv_empty[s0]);
+                        release(&bars.pv_empty[s0 + 1]);
+                        rp.advance(CB);
+                        rp.advance(CB);
+                    }
+                    if (!ok) break;
+                    tc::commit_elect(smem_u32(&bars.pv_done));
+                    if (lane == 0) GBMLA_TRACE_EVENT(5, t);
+                    if (tail) ++n_tail;
+                }
             }
-            if (!ok) {
+            if (!ok && lane == 0) {
                 record_status(a.status, kStatusTimeout);
                 ss.abort = 1;
             }
-            // drain: every MMA this thread issued has completed before TMEM is freed
-            tc::commit(smem_u32(&bars.drain));
-            if (!mbar_wait(smem_u32(&bars.drain), 0, lim_ns)) record_status(a.status, kStatusTimeout);
+            // drain: every MMA this warp issued has completed before TMEM is freed
+            tc::commit_elect(smem_u32(drain));
+            if (!__all_sync(0xffffffffu, mbar_wait(smem_u32(drain), 0, lim_ns)) && lane == 0)
+                record_status(a.status, kStatusTimeout);
         }
     } else {
         // ================================================================ softmax / epilogue
@@ -805,19 +856,19 @@ __global__ void __maxnreg__(128)
         c.lane = lane;
         c.tid = tid;
         c.quarter = warp & 3;                 // TMEM lane quarter this warp may access
-        c.half = (warp - 2) >> 2;             // which column blocks it owns: half, half+3, ...
+        c.half = (warp - 4) >> 2;             // which column blocks it owns: half, half+3, ...
         c.tok = c.quarter * 32 + lane;        // token row of the tile
-        c.n_own = c.half < NB ? (NB - c.half + 2) / 3 : 0;
+        c.n_own = c.half < N / 16 ? (N / 16 - c.half + 2) / 3 : 0;
         c.group = group;
         c.part = part;
         c.nrc = nrc;
         c.ncc = ncc;
-        c.cs = CS;
+        c.cs = CB;
         c.n_items = n_items;
         c.lane_base = static_cast<uint32_t>(c.quarter * 32) << 16;
         c.tmem = tmem;
         c.o_col0 = o_col0;
-        c.ring = ring;
+        c.ring = ring_b;
         c.p_buf = p_buf;
         c.lim_ns = lim_ns;
         c.t_begin = t_begin;
@@ -848,14 +899,14 @@ cudaError_t get_encoder()
     return cudaSuccess;
 }
 
-// 3-d map over one cache: (columns, tokens per block, blocks), box 64 x 64 x 1, SW128.
+// 3-d map over one cache: (columns, tokens per block, blocks), box 64 x box_rows x 1, SW128.
 cudaError_t encode_cache_map(CUtensorMap *m, const void *base, int cols, int64_t tok_stride, int64_t blk_stride,
-                             int tokens_per_block, int blocks)
+                             int tokens_per_block, int blocks, int box_rows)
 {
     cuuint64_t dims[3] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(tokens_per_block),
                           static_cast<cuuint64_t>(blocks)};
     cuuint64_t strides[2] = {static_cast<cuuint64_t>(tok_stride) * 2, static_cast<cuuint64_t>(blk_stride) * 2};
-    cuuint32_t box[3] = {64, static_cast<cuuint32_t>(kHalf), 1};
+    cuuint32_t box[3] = {64, static_cast<cuuint32_t>(box_rows), 1};
     cuuint32_t es[3] = {1, 1, 1};
     CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, es,
                           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -873,8 +924,9 @@ cudaError_t launch_cfg(const AttnArgs &a, int groups, cudaStream_t st)
     const int tpb = paged ? c.page_size : c.capacity;
     const int blocks = paged ? c.num_pages : a.batch;
     CUtensorMap mc, mr, mq;
-    if ((e = encode_cache_map(&mc, c.c_kv, a.rank, c.c_tok, c.c_blk, tpb, blocks)) != cudaSuccess) return e;
-    if ((e = encode_cache_map(&mr, c.k_rope, a.d_rope, c.r_tok, c.r_blk, tpb, blocks)) != cudaSuccess) return e;
+    const int box_rows = paged ? kHalf : kTile;
+    if ((e = encode_cache_map(&mc, c.c_kv, a.rank, c.c_tok, c.c_blk, tpb, blocks, box_rows)) != cudaSuccess) return e;
+    if ((e = encode_cache_map(&mr, c.k_rope, a.d_rope, c.r_tok, c.r_blk, tpb, blocks, box_rows)) != cudaSuccess) return e;
     {
         const int K = a.rank + a.d_rope;
         cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(a.batch) * a.q_len * a.num_heads};
@@ -889,19 +941,25 @@ cudaError_t launch_cfg(const AttnArgs &a, int groups, cudaStream_t st)
     const int ncc = a.rank / 64;
     const int q_bytes = (((ncc + 1) * N * 128) + 1023) & ~1023;
     const int p_bytes = (N / 16) * kTile * 32;
-    const int fixed = 1024 /*alignment slack*/ + q_bytes + kChunkBytes /*positional keys*/;
+    const int fixed = 1024 /*alignment slack*/ + q_bytes;
     int dev = 0, optin = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
     const int static_bytes = static_cast<int>(sizeof(Bars) + sizeof(Shared<N>) + 32 * 8) + 128;
     int slots = (optin - static_bytes - fixed - p_bytes) / kChunkBytes;
     if (slots > kMaxSlots) slots = kMaxSlots;
-    if (const char *env = getenv("GBMLA_TC_MAX_SLOTS")) {  // testing aid: a smaller ring
+    if (const char *env = getenv("GBMLA_TC_MAX_SLOTS")) {  // testing aid: smaller rings
         const int cap = atoi(env);
         if (cap >= 4 && cap < slots) slots = cap;
     }
-    slots &= ~1;
     if (slots < 4) return cudaErrorInvalidConfiguration;
+    // the PV ring (refilled from L2) gets two or four slots, the QK ring the rest
+    int pv_slots = slots >= 9 ? 4 : 2;
+    if (const char *env = getenv("GBMLA_TC_PV_SLOTS")) {  // testing aid
+        const int v = atoi(env) & ~1;
+        if (v >= 2 && v <= slots - 2) pv_slots = v;
+    }
+    const int qk_slots = slots - pv_slots;
     const size_t smem = static_cast<size_t>(fixed) + static_cast<size_t>(slots) * kChunkBytes + p_bytes;
     if ((e = cudaFuncSetAttribute(attn_tc_kernel<N, CL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   static_cast<int>(smem))) != cudaSuccess)
@@ -918,7 +976,8 @@ cudaError_t launch_cfg(const AttnArgs &a, int groups, cudaStream_t st)
     t.paged = paged;
     t.bt_stride = c.bt_stride;
     t.num_pages = c.num_pages;
-    t.c_slots = slots;
+    t.qk_slots = qk_slots;
+    t.pv_slots = pv_slots;
     t.scale_log2 = a.sm_scale * 1.4426950408889634f;
     t.kv_len = a.kv_len;
     t.block_table = c.block_table;

@@ -79,6 +79,44 @@ __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint6
         : "memory");
 }
 
+// Warp-collective forms: the whole warp executes them converged and one
+// elected lane issues.  A lone lane running the issue loop pays a large
+// per-iteration cost for every branch; a converged warp does not.
+__device__ __forceinline__ void mma_bf16_elect(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                               uint32_t accumulate)
+{
+    asm volatile(
+        "{\n .reg .pred p, e;\n elect.sync _|e, 0xffffffff;\n setp.ne.b32 p, %4, 0;\n"
+        " @e tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+__device__ __forceinline__ void commit_elect(uint32_t mbar)
+{
+    asm volatile(
+        "{\n .reg .pred e;\n elect.sync _|e, 0xffffffff;\n"
+        " @e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n}\n" ::"r"(mbar)
+        : "memory");
+}
+
+__device__ __forceinline__ void commit_multicast_elect(uint32_t mbar, uint16_t cta_mask)
+{
+    asm volatile(
+        "{\n .reg .pred e;\n elect.sync _|e, 0xffffffff;\n"
+        " @e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;\n}\n" ::"r"(
+            mbar),
+        "h"(cta_mask)
+        : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_elect(uint32_t mbar)
+{
+    asm volatile(
+        "{\n .reg .pred e;\n elect.sync _|e, 0xffffffff;\n @e mbarrier.arrive.shared::cta.b64 _, [%0];\n}\n" ::"r"(mbar)
+        : "memory");
+}
+
 // Arrive once on the mbarrier when every MMA this thread issued so far has
 // completed (and its smem operands may be overwritten).
 __device__ __forceinline__ void commit(uint32_t mbar)
