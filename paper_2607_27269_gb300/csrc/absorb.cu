@@ -3,25 +3,9 @@
 // query rotated to its own position (Sec. 3.1).
 #include "common.cuh"
 #include "internal.h"
-#include "simt_gemm.cuh"
 
 namespace gbmla {
 namespace {
-
-// Rows of group g: (bi, hh) with bi = b*q_len + i and head g*hpg + hh.
-__global__ void __launch_bounds__(256) absorb_gemm_kernel(int rows_g, int H, int hpg, int d_nope, int rank,
-                                                         int ld_out, const uint16_t *__restrict__ q_nope,
-                                                         const uint16_t *__restrict__ w_uk, uint16_t *q_abs)
-{
-    const int g = blockIdx.z;
-    auto grow = [=](int m) { return static_cast<int64_t>(m / hpg) * H + g * hpg + m % hpg; };
-    const uint16_t *w = w_uk + static_cast<int64_t>(g) * d_nope * rank;
-    simt_gemm_64x64(
-        blockIdx.x * 64, blockIdx.y * 64, rows_g, rank, d_nope,
-        [=](int m, int k) { return bf16_bits_to_float(q_nope[grow(m) * d_nope + k]); },
-        [=](int n, int k) { return bf16_bits_to_float(w[static_cast<int64_t>(k) * rank + n]); },
-        [=](int m, int n, float v) { q_abs[grow(m) * ld_out + n] = __bfloat16_as_ushort(__float2bfloat16_rn(v)); });
-}
 
 // One block per (b, i): angles of position kv_len[b] - q_len + i are shared
 // by all heads.
@@ -55,14 +39,24 @@ cudaError_t launch_absorb(const mla_dims &d, int batch, int q_len, const void *q
                           const int32_t *kv_len, const void *w_uk, void *q_abs, unsigned *status,
                           cudaStream_t st)
 {
-    (void)status;
     const int H = d.num_heads, G = d.num_kv_groups, hpg = H / G;
-    const int rows_g = batch * q_len * hpg;
-    dim3 grid((rows_g + 63) / 64, (d.rank + 63) / 64, G);
-    absorb_gemm_kernel<<<grid, 256, 0, st>>>(rows_g, H, hpg, d.d_nope, d.rank, d.rank + d.d_rope,
-                                             static_cast<const uint16_t *>(q_nope),
-                                             static_cast<const uint16_t *>(w_uk), static_cast<uint16_t *>(q_abs));
-    cudaError_t e = cudaGetLastError();
+    // rows of group g: (b, i, head g*hpg + hh); q_lat = q_nope W_UK[g] (W_UK: d_nope x rank)
+    GroupGemm p;
+    p.M = batch * q_len * hpg;
+    p.N = d.rank;
+    p.K = d.d_nope;
+    p.G = G;
+    p.hpg = hpg;
+    p.blk = H;
+    p.A = q_nope;
+    p.a_f32 = 0;
+    p.lda = d.d_nope;
+    p.B = w_uk;
+    p.b_nmajor = 1;
+    p.C = q_abs;
+    p.ldc = d.rank + d.d_rope;
+    p.status = status;
+    cudaError_t e = launch_group_gemm(p, st);
     if (e != cudaSuccess) return e;
     absorb_rope_kernel<<<batch * q_len, 256, 0, st>>>(q_len, H, d.rank, d.d_rope, d.rope_style, d.rope_base, kv_len,
                                                       static_cast<const uint16_t *>(q_pe),

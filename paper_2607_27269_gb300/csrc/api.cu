@@ -233,6 +233,7 @@ mla_status mla_absorb_q(const mla_dims *dims, int32_t batch, int32_t q_len, cons
     if (batch < 0 || q_len < 1 || q_len > 16) return MLA_ERR_INVALID_ARG;
     if (batch == 0) return MLA_OK;
     if (!q_nope || !q_pe || !kv_len || !w_uk || !q_abs) return MLA_ERR_INVALID_ARG;
+    if (!aligned16(q_nope) || !aligned16(w_uk) || !aligned16(q_abs)) return MLA_ERR_INVALID_ARG;
     if (static_cast<int64_t>(batch) * q_len > (1 << 30)) return MLA_ERR_UNSUPPORTED;
     unsigned *status = nullptr;
     if ((s = device_info(&status, nullptr)) != MLA_OK) return s;
@@ -302,8 +303,11 @@ mla_status mla_out_proj(const mla_dims *dims, int32_t batch, int32_t q_len, cons
     if (batch == 0) return MLA_OK;
     if (!o_lat || !w_uv || !o) return MLA_ERR_INVALID_ARG;
     if (w_o && dims->hidden > 0 && !out) return MLA_ERR_INVALID_ARG;
-    if ((s = device_info(nullptr, nullptr)) != MLA_OK) return s;
-    return from_cuda(launch_out_proj(*dims, batch, q_len, o_lat, w_uv, w_o, o, out,
+    if (!aligned16(o_lat) || !aligned16(w_uv) || !aligned16(o)) return MLA_ERR_INVALID_ARG;
+    if (w_o && dims->hidden > 0 && (!aligned16(w_o) || !aligned16(out))) return MLA_ERR_INVALID_ARG;
+    unsigned *status = nullptr;
+    if ((s = device_info(&status, nullptr)) != MLA_OK) return s;
+    return from_cuda(launch_out_proj(*dims, batch, q_len, o_lat, w_uv, w_o, o, out, status,
                                      static_cast<cudaStream_t>(stream)));
 }
 

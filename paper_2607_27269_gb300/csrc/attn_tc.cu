@@ -76,7 +76,8 @@ struct __align__(8) Bars {
     uint64_t pv_full[kMaxSlots], pv_empty[kMaxSlots];  // PV ring: latent chunks again
     uint64_t q_full, q_free;
     uint64_t s_full[2], s_free[2];
-    uint64_t p_full, pv_done, o_free, drain_qk, drain_pv;
+    uint64_t p_full[2], pv_done[2];  // per P buffer: P(t) published / PV(t) completed, t & 1
+    uint64_t o_free, drain_qk, drain_pv;
     // Tail tile handshake per r-chunk m: the PV warp (which waits on its
     // ring in strict order) reports that chunks 2m, 2m+1 landed (zready);
     // the softmax warps clear their rows past the end (zdone).
@@ -253,17 +254,31 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const float (&v)[16])
 struct SmCtx {
     int lane, tid, quarter, half, tok, n_own, group, part, nrc, ncc, cs, n_items;
     uint32_t lane_base, tmem, o_col0;
-    unsigned char *ring, *p_buf;
+    unsigned char *ring, *p_buf;  // p_buf: two P buffers of NB x [128 tok x 32 B]
     uint64_t lim_ns;
     int64_t t_begin, t_end;
 };
 
 // The whole warp waits; a failure marks sm_fail, which the softmax
 // warps read only after their next named barrier, so they all leave together.
+#ifdef GBMLA_TRACE
+__shared__ unsigned long long s_sm_wait_cyc;
+#endif
 template <int N>
 __device__ __forceinline__ void sm_wait(const SmCtx &c, const TcArgs &a, Shared<N> &ss, uint64_t *bar,
                                         uint32_t parity)
 {
+#ifdef GBMLA_TRACE
+    const long long w0 = clock64();
+    struct Acc {
+        long long t0;
+        int lane;
+        __device__ ~Acc()
+        {
+            if (lane == 0) atomicAdd(&s_sm_wait_cyc, static_cast<unsigned long long>(clock64() - t0));
+        }
+    } acc{w0, c.lane};
+#endif
     if (!__all_sync(0xffffffffu, mbar_wait(smem_u32(bar), parity, c.lim_ns)) && c.lane == 0) {
         record_status(a.status, kStatusTimeout);
         atomicOr(&ss.sm_fail, 1);
@@ -308,7 +323,7 @@ template <int N, int KOWN>
 __device__ __forceinline__ void sm_epilogue(const SmCtx &c, const TcArgs &a, Shared<N> &ss, Bars &bars,
                                             float (&l_part)[KOWN][16], int b, int64_t t_end_seg)
 {
-    sm_wait<N>(c, a, ss, &bars.pv_done, static_cast<uint32_t>(t_end_seg & 1));
+    sm_wait<N>(c, a, ss, &bars.pv_done[t_end_seg & 1], static_cast<uint32_t>((t_end_seg >> 1) & 1));
     named_sync_softmax();
     if (ss.sm_fail) return;
     tc::fence_after_sync();
@@ -450,14 +465,18 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
             }
         }
         named_sync_softmax();
-        // ---- P is rewritten and O^T rescaled only once PV(t-1) has completed
-        if (!first) {
-            if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(7, t);
-            sm_wait<N>(c, a, ss, &bars.pv_done, static_cast<uint32_t>((t - 1) & 1));
-            if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(8, t);
-            named_sync_softmax();
-            if (ss.sm_fail) break;
-            tc::fence_after_sync();
+        // ---- P(t) goes to buffer t & 1, free again once PV(t-2) has completed;
+        // O^T is rescaled (rarely: only when a base moves) once PV(t-1) has
+        // completed.  Each wait is on the next phase of its barrier.
+        if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(7, t);
+        if (t >= 2) sm_wait<N>(c, a, ss, &bars.pv_done[t & 1], static_cast<uint32_t>(((t - 2) >> 1) & 1));
+        if (ss.any_rescale)  // never on a sequence's first tile
+            sm_wait<N>(c, a, ss, &bars.pv_done[(t - 1) & 1], static_cast<uint32_t>(((t - 1) >> 1) & 1));
+        if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(8, t);
+        named_sync_softmax();
+        if (ss.sm_fail) break;
+        tc::fence_after_sync();
+        {
             if (ss.any_rescale) {
 #pragma unroll
                 for (int ob = 0; ob < KOWN; ++ob) {
@@ -498,7 +517,7 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
                     l_part[ob][e + 1] += __high2float(pb);
                     pk[e / 2] = *reinterpret_cast<const uint32_t *>(&pb);
                 }
-                unsigned char *row = c.p_buf + cb * (kTile * 32) + c.tok * 32;
+                unsigned char *row = c.p_buf + (t & 1) * (N / 16) * (kTile * 32) + cb * (kTile * 32) + c.tok * 32;
                 const int sw = (c.tok >> 2) & 1;
                 *reinterpret_cast<uint4 *>(row + (sw * 16)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
                 *reinterpret_cast<uint4 *>(row + ((1 ^ sw) * 16)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
@@ -510,7 +529,7 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
         tc::fence_proxy_async_smem();
         tc::fence_before_sync();
         __syncwarp();
-        if (c.lane == 0) tc::mbar_arrive(smem_u32(&bars.p_full));
+        if (c.lane == 0) tc::mbar_arrive(smem_u32(&bars.p_full[t & 1]));
         if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(9, t);
         // ---- tail tile: rows past the sequence end in the PV copy of the
         // latent chunks are cleared, so stale or uninitialised bytes never meet
@@ -562,7 +581,7 @@ __global__ void __maxnreg__(128)
     unsigned char *q_buf = smem;                                          // nqc x [N x 128 B]
     unsigned char *ring_a = q_buf + ((nqc * N * 128 + 1023) & ~1023);     // CA x [128 x 128 B]
     unsigned char *ring_b = ring_a + CA * kChunkBytes;                    // CB x [128 x 128 B]
-    unsigned char *p_buf = ring_b + CB * kChunkBytes;                     // NB x [128 tok x 32 B]
+    unsigned char *p_buf = ring_b + CB * kChunkBytes;                     // 2 x NB x [128 tok x 32 B]
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int group = blockIdx.x, part = blockIdx.y;
@@ -593,8 +612,10 @@ __global__ void __maxnreg__(128)
             mbar_init(&bars.s_full[i], 1);
             mbar_init(&bars.s_free[i], kSoftmaxWarps);
         }
-        mbar_init(&bars.p_full, kSoftmaxWarps);
-        mbar_init(&bars.pv_done, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&bars.p_full[i], kSoftmaxWarps);
+            mbar_init(&bars.pv_done[i], 1);
+        }
         mbar_init(&bars.o_free, kSoftmaxWarps);
         mbar_init(&bars.drain_qk, 1);
         mbar_init(&bars.drain_pv, 1);
@@ -604,6 +625,7 @@ __global__ void __maxnreg__(128)
         }
 #ifdef GBMLA_TRACE
         s_trace_count = 0;
+        s_sm_wait_cyc = 0;
 #endif
         ss.need_max = 0;
         ss.any_rescale = 0;
@@ -751,8 +773,18 @@ __global__ void __maxnreg__(128)
             w.init(a.kv_len, a.batch, a.q_len, a.max_kv, t_begin, t_end);
             RingPos rp{0, 0};
             bool ok = true;
+#ifdef GBMLA_TRACE
+            long long wait_cyc = 0;
+            const long long loop_t0 = clock64();
+#endif
             auto wait = [&](uint64_t *bar, uint32_t parity) {
+#ifdef GBMLA_TRACE
+                const long long w0 = clock64();
+#endif
                 if (ok) ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(bar), parity, lim_ns));
+#ifdef GBMLA_TRACE
+                wait_cyc += clock64() - w0;
+#endif
                 return ok;
             };
             // a consumed slot is handed back to every CTA of the cluster
@@ -803,7 +835,7 @@ __global__ void __maxnreg__(128)
                 int seg = -1, n_tail = 0;
                 for (int t = 0; t < n_items && ok; ++t, w.next()) {
                     if (any_abort()) break;
-                    if (!wait(&bars.p_full, t & 1)) break;
+                    if (!wait(&bars.p_full[t & 1], (t >> 1) & 1)) break;
                     if (lane == 0) GBMLA_TRACE_EVENT(4, t);
                     bool first_pv = false;
                     if (w.first()) {
@@ -824,11 +856,12 @@ __global__ void __maxnreg__(128)
                         }
                         tc::fence_after_sync();
                         const uint32_t cb = ring_base + s0 * kChunkBytes;
+                        const uint32_t pb = p_base + (t & 1) * (N / 16) * (kTile * 32);
                         const uint32_t d_o = tmem + o_col0 + m * N;
 #pragma unroll
                         for (int kk = 0; kk < kTile / 16; ++kk)
                             tc::mma_bf16_elect(d_o, with_addr(dc, cb + kk * 16 * 128),
-                                               with_addr(dp, p_base + kk * 16 * 32), id_pv,
+                                               with_addr(dp, pb + kk * 16 * 32), id_pv,
                                                (first_pv && kk == 0) ? 0u : 1u);
                         release(&bars.pv_empty[s0]);
                         release(&bars.pv_empty[s0 + 1]);
@@ -836,7 +869,7 @@ __global__ void __maxnreg__(128)
                         rp.advance(CB);
                     }
                     if (!ok) break;
-                    tc::commit_elect(smem_u32(&bars.pv_done));
+                    tc::commit_elect(smem_u32(&bars.pv_done[t & 1]));
                     if (lane == 0) GBMLA_TRACE_EVENT(5, t);
                     if (tail) ++n_tail;
                 }
@@ -845,6 +878,12 @@ __global__ void __maxnreg__(128)
                 record_status(a.status, kStatusTimeout);
                 ss.abort = 1;
             }
+#ifdef GBMLA_TRACE
+            if (lane == 0) {
+                GBMLA_TRACE_EVENT(is_qk ? 20 : 21, wait_cyc);
+                GBMLA_TRACE_EVENT(is_qk ? 22 : 23, clock64() - loop_t0);
+            }
+#endif
             // drain: every MMA this warp issued has completed before TMEM is freed
             tc::commit_elect(smem_u32(drain));
             if (!__all_sync(0xffffffffu, mbar_wait(smem_u32(drain), 0, lim_ns)) && lane == 0)
@@ -873,7 +912,17 @@ __global__ void __maxnreg__(128)
         c.lim_ns = lim_ns;
         c.t_begin = t_begin;
         c.t_end = t_end;
+#ifdef GBMLA_TRACE
+        const long long sm_t0 = clock64();
+#endif
         softmax_role<N>(c, a, ss, bars);
+#ifdef GBMLA_TRACE
+        named_sync_softmax();
+        if (tid == kSoftmaxBase) {
+            GBMLA_TRACE_EVENT(24, static_cast<int64_t>(s_sm_wait_cyc / kSoftmaxWarps));
+            GBMLA_TRACE_EVENT(25, clock64() - sm_t0);
+        }
+#endif
     }
 
     tc::fence_before_sync();
@@ -940,7 +989,7 @@ cudaError_t launch_cfg(const AttnArgs &a, int groups, cudaStream_t st)
     }
     const int ncc = a.rank / 64;
     const int q_bytes = (((ncc + 1) * N * 128) + 1023) & ~1023;
-    const int p_bytes = (N / 16) * kTile * 32;
+    const int p_bytes = 2 * (N / 16) * kTile * 32;  // two P buffers
     const int fixed = 1024 /*alignment slack*/ + q_bytes;
     int dev = 0, optin = 0;
     cudaGetDevice(&dev);

@@ -55,7 +55,26 @@ cudaError_t launch_combine(int batch, int q_len, int num_heads, int rank, int ma
                            float *lse, cudaStream_t st);
 
 cudaError_t launch_out_proj(const mla_dims &d, int batch, int q_len, const float *o_lat, const void *w_uv,
-                            const void *w_o, void *o, void *out, cudaStream_t st);
+                            const void *w_o, void *o, void *out, unsigned *status, cudaStream_t st);
+
+// Grouped GEMM of the projections: for each group g < G and row m < M,
+// C[phys(g, m), n] = sum_k A[phys(g, m), k] B_g(n, k) (bf16 result), with
+// phys(g, m) = (m / hpg) * blk + g * hpg + m % hpg.  A is fp32 or bf16 with
+// row stride lda; B_g(n, k) = B[g N K + n K + k] (K-major) or B[g K N + k N + n]
+// (N-major), bf16.  K and N are multiples of 8; A, B and C 16-byte aligned.
+struct GroupGemm {
+    int M, N, K, G;
+    int hpg, blk;
+    const void *A;
+    int a_f32;
+    int64_t lda;
+    const void *B;
+    int b_nmajor;
+    void *C;
+    int64_t ldc;
+    unsigned *status;
+};
+cudaError_t launch_group_gemm(const GroupGemm &p, cudaStream_t st);
 
 cudaError_t launch_selftest_wait(int64_t limit_ns, unsigned *status, cudaStream_t st);
 
