@@ -39,6 +39,11 @@ constexpr int kSoftmaxWarps = 12;
 constexpr int kSoftmaxBase = 128;           // first softmax thread (after two producer and two MMA warps)
 constexpr int kThreads = kSoftmaxBase + 32 * kSoftmaxWarps;
 
+// P buffers: two (softmax of tile t overlaps PV(t-1)) where shared memory
+// allows; one for 80-row groups, whose queries leave room for little else.
+template <int N>
+constexpr int kPBufs = N >= 80 ? 1 : 2;
+
 // Optional event trace of the first CTA (compiled only with -DGBMLA_TRACE):
 // (globaltimer ns, event code, argument) triples in a caller buffer, set by
 // mla_debug_trace().  Used to read the per-tile timeline of the roles.
@@ -76,7 +81,7 @@ struct __align__(8) Bars {
     uint64_t pv_full[kMaxSlots], pv_empty[kMaxSlots];  // PV ring: latent chunks again
     uint64_t q_full, q_free;
     uint64_t s_full[2], s_free[2];
-    uint64_t p_full[2], pv_done[2];  // per P buffer: P(t) published / PV(t) completed, t & 1
+    uint64_t p_full[2], pv_done[2];  // per P buffer (t % NP): P(t) published / PV(t) completed
     uint64_t o_free, drain_qk, drain_pv;
     // Tail tile handshake per r-chunk m: the PV warp (which waits on its
     // ring in strict order) reports that chunks 2m, 2m+1 landed (zready);
@@ -254,7 +259,7 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const float (&v)[16])
 struct SmCtx {
     int lane, tid, quarter, half, tok, n_own, group, part, nrc, ncc, cs, n_items;
     uint32_t lane_base, tmem, o_col0;
-    unsigned char *ring, *p_buf;  // p_buf: two P buffers of NB x [128 tok x 32 B]
+    unsigned char *ring, *p_buf;  // p_buf: NP buffers of NB x [128 tok x 32 B]
     uint64_t lim_ns;
     int64_t t_begin, t_end;
 };
@@ -323,7 +328,7 @@ template <int N, int KOWN>
 __device__ __forceinline__ void sm_epilogue(const SmCtx &c, const TcArgs &a, Shared<N> &ss, Bars &bars,
                                             float (&l_part)[KOWN][16], int b, int64_t t_end_seg)
 {
-    sm_wait<N>(c, a, ss, &bars.pv_done[t_end_seg & 1], static_cast<uint32_t>((t_end_seg >> 1) & 1));
+    sm_wait<N>(c, a, ss, &bars.pv_done[t_end_seg % kPBufs<N>], static_cast<uint32_t>((t_end_seg / kPBufs<N>) & 1));
     named_sync_softmax();
     if (ss.sm_fail) return;
     tc::fence_after_sync();
@@ -465,13 +470,14 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
             }
         }
         named_sync_softmax();
-        // ---- P(t) goes to buffer t & 1, free again once PV(t-2) has completed;
-        // O^T is rescaled (rarely: only when a base moves) once PV(t-1) has
-        // completed.  Each wait is on the next phase of its barrier.
+        // ---- P(t) goes to buffer t % NP, free again once PV(t - NP) has
+        // completed; O^T is rescaled (rarely: only when a base moves) once
+        // PV(t-1) has completed.  Each wait is on the next phase of its barrier.
+        constexpr int NP = kPBufs<N>;
         if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(7, t);
-        if (t >= 2) sm_wait<N>(c, a, ss, &bars.pv_done[t & 1], static_cast<uint32_t>(((t - 2) >> 1) & 1));
+        if (t >= NP) sm_wait<N>(c, a, ss, &bars.pv_done[t % NP], static_cast<uint32_t>(((t - NP) / NP) & 1));
         if (ss.any_rescale)  // never on a sequence's first tile
-            sm_wait<N>(c, a, ss, &bars.pv_done[(t - 1) & 1], static_cast<uint32_t>(((t - 1) >> 1) & 1));
+            sm_wait<N>(c, a, ss, &bars.pv_done[(t - 1) % NP], static_cast<uint32_t>(((t - 1) / NP) & 1));
         if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(8, t);
         named_sync_softmax();
         if (ss.sm_fail) break;
@@ -517,7 +523,7 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
                     l_part[ob][e + 1] += __high2float(pb);
                     pk[e / 2] = *reinterpret_cast<const uint32_t *>(&pb);
                 }
-                unsigned char *row = c.p_buf + (t & 1) * (N / 16) * (kTile * 32) + cb * (kTile * 32) + c.tok * 32;
+                unsigned char *row = c.p_buf + (t % kPBufs<N>) * (N / 16) * (kTile * 32) + cb * (kTile * 32) + c.tok * 32;
                 const int sw = (c.tok >> 2) & 1;
                 *reinterpret_cast<uint4 *>(row + (sw * 16)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
                 *reinterpret_cast<uint4 *>(row + ((1 ^ sw) * 16)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
@@ -529,7 +535,7 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
         tc::fence_proxy_async_smem();
         tc::fence_before_sync();
         __syncwarp();
-        if (c.lane == 0) tc::mbar_arrive(smem_u32(&bars.p_full[t & 1]));
+        if (c.lane == 0) tc::mbar_arrive(smem_u32(&bars.p_full[t % kPBufs<N>]));
         if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(9, t);
         // ---- tail tile: rows past the sequence end in the PV copy of the
         // latent chunks are cleared, so stale or uninitialised bytes never meet
@@ -581,7 +587,7 @@ __global__ void __maxnreg__(128)
     unsigned char *q_buf = smem;                                          // nqc x [N x 128 B]
     unsigned char *ring_a = q_buf + ((nqc * N * 128 + 1023) & ~1023);     // CA x [128 x 128 B]
     unsigned char *ring_b = ring_a + CA * kChunkBytes;                    // CB x [128 x 128 B]
-    unsigned char *p_buf = ring_b + CB * kChunkBytes;                     // 2 x NB x [128 tok x 32 B]
+    unsigned char *p_buf = ring_b + CB * kChunkBytes;                     // NP x NB x [128 tok x 32 B]
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int group = blockIdx.x, part = blockIdx.y;
@@ -835,7 +841,7 @@ __global__ void __maxnreg__(128)
                 int seg = -1, n_tail = 0;
                 for (int t = 0; t < n_items && ok; ++t, w.next()) {
                     if (any_abort()) break;
-                    if (!wait(&bars.p_full[t & 1], (t >> 1) & 1)) break;
+                    if (!wait(&bars.p_full[t % kPBufs<N>], (t / kPBufs<N>) & 1)) break;
                     if (lane == 0) GBMLA_TRACE_EVENT(4, t);
                     bool first_pv = false;
                     if (w.first()) {
@@ -856,7 +862,7 @@ __global__ void __maxnreg__(128)
                         }
                         tc::fence_after_sync();
                         const uint32_t cb = ring_base + s0 * kChunkBytes;
-                        const uint32_t pb = p_base + (t & 1) * (N / 16) * (kTile * 32);
+                        const uint32_t pb = p_base + (t % kPBufs<N>) * (N / 16) * (kTile * 32);
                         const uint32_t d_o = tmem + o_col0 + m * N;
 #pragma unroll
                         for (int kk = 0; kk < kTile / 16; ++kk)
@@ -869,7 +875,7 @@ __global__ void __maxnreg__(128)
                         rp.advance(CB);
                     }
                     if (!ok) break;
-                    tc::commit_elect(smem_u32(&bars.pv_done[t & 1]));
+                    tc::commit_elect(smem_u32(&bars.pv_done[t % kPBufs<N>]));
                     if (lane == 0) GBMLA_TRACE_EVENT(5, t);
                     if (tail) ++n_tail;
                 }
@@ -989,7 +995,7 @@ cudaError_t launch_cfg(const AttnArgs &a, int groups, cudaStream_t st)
     }
     const int ncc = a.rank / 64;
     const int q_bytes = (((ncc + 1) * N * 128) + 1023) & ~1023;
-    const int p_bytes = 2 * (N / 16) * kTile * 32;  // two P buffers
+    const int p_bytes = kPBufs<N> * (N / 16) * kTile * 32;
     const int fixed = 1024 /*alignment slack*/ + q_bytes;
     int dev = 0, optin = 0;
     cudaGetDevice(&dev);
@@ -1003,7 +1009,7 @@ cudaError_t launch_cfg(const AttnArgs &a, int groups, cudaStream_t st)
     }
     if (slots < 4) return cudaErrorInvalidConfiguration;
     // the PV ring (refilled from L2) gets two or four slots, the QK ring the rest
-    int pv_slots = slots >= 9 ? 4 : 2;
+    int pv_slots = slots >= 6 ? 4 : 2;
     if (const char *env = getenv("GBMLA_TC_PV_SLOTS")) {  // testing aid
         const int v = atoi(env) & ~1;
         if (v >= 2 && v <= slots - 2) pv_slots = v;
