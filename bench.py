@@ -48,6 +48,8 @@ def parse_args(argv=None):
     p.add_argument("--no-graph", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--seed", type=int, default=0)
+    p.add_argument("--attn-launches", type=int, default=0,
+                   help="profiling aid: one full step, then this many attention launches alone; no timing")
     return p.parse_args(argv)
 
 
@@ -333,6 +335,28 @@ def load_peaks():
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "source": "fallback"}
 
 
+def run_attn_only(args, local):
+    """Profiling aid (for ncu captures of one kernel on one copy of the
+    workload): one full decode step, then `--attn-launches` launches of the
+    attention kernel alone.  Prints one JSON line with the device status."""
+    import torch
+    from paper_2607_27269_gb300 import abi
+    from paper_2607_27269_gb300 import workloads as wl
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    w = wl.make(wl.SHAPES[args.workload], seed=args.seed)
+    d = abi.to_device(w, dev)
+    st = abi.DecodeStep(d.dims, d.cache, d.batch, d.q_len, d.max_kv_len, args.num_splits)
+    st(d.q_nope, d.q_pe, d.kv_len, d.w_uk, d.w_uv, d.w_o, c_new=d.c_new, kr_new=d.kr_new, start_pos=d.start_pos)
+    for _ in range(args.attn_launches):
+        abi.decode_attn(d.dims, d.cache, d.kv_len, d.max_kv_len, st.q_abs, st.o_part, st.lse_part, st.num_splits)
+    torch.cuda.synchronize(dev)
+    code = abi.check_status()
+    return {"profile": "attn_only", "workload": w.shape.name, "launches": args.attn_launches,
+            "num_splits": st.num_splits, "cache_bytes": w.cache_bytes, "status": abi.status_name(code)}, code
+
+
 # ---------------------------------------------------------------- the oracle on the host
 
 def oracle_sample(w, budget_s: float = 20.0):
@@ -424,6 +448,10 @@ def main(argv=None):
             import torch
             torch.cuda.set_device(local)
             dist.init_process_group("nccl")
+    if args.attn_launches > 0:
+        line, code = run_attn_only(args, local)
+        print(json.dumps(line), flush=True)
+        return 0 if code == 0 else 1
     if args.impl == "reference":
         line = run_reference(args, rank, world)
         if line is not None:

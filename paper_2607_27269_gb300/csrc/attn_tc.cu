@@ -687,6 +687,7 @@ __global__ void __maxnreg__(128)
             bool has = (kind == kQK || kind == kPV) ? c < total : kind == kQuery;
             bool ok = true;
             uint64_t wait_t0 = 0;
+            const uint64_t pol_keep = tc::policy_evict_last(), pol_drop = tc::policy_evict_first();
             uint32_t wbar = 0, fbar = 0, dst = 0;
             if (kind == kQK) {
                 wbar = smem_u32(&bars.qk_empty[slot]);
@@ -736,12 +737,16 @@ __global__ void __maxnreg__(128)
                             if (lane == 0 && warp == 0) GBMLA_TRACE_EVENT(1, c);
                             tc::mbar_arrive_expect_tx(fbar, L.bytes);
                             if (c % CL == rank_in_cluster) {
+                                // the QK pass keeps latent lines in L2 for the PV pass, which reads
+                                // them a last time; the positional keys are read once
+                                const uint64_t pol = (kind == kQK && !keys) ? pol_keep : pol_drop;
                                 for (int h = 0; h < L.nh; ++h) {
                                     if (CL > 1)
-                                        tc::tma_load_3d_multicast(dst + h * kHalf * 128, map, col, L.tok0[h],
-                                                                  L.blk[h], fbar, kMask);
+                                        tc::tma_load_3d_multicast_hint(dst + h * kHalf * 128, map, col, L.tok0[h],
+                                                                       L.blk[h], fbar, kMask, pol);
                                     else
-                                        tc::tma_load_3d(dst + h * kHalf * 128, map, col, L.tok0[h], L.blk[h], fbar);
+                                        tc::tma_load_3d_hint(dst + h * kHalf * 128, map, col, L.tok0[h], L.blk[h],
+                                                             fbar, pol);
                                 }
                             }
                             c += ring_len;
