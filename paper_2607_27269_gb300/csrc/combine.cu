@@ -32,10 +32,13 @@ __global__ void __launch_bounds__(256) combine_kernel(int batch, int q_len, int 
     const int row = blockIdx.x * rpb + threadIdx.x / tpr;
     const int part = threadIdx.x % tpr;
     if (row >= rows) return;
+    // a partition is empty only when there are fewer tiles than partitions
+    const bool may_be_empty = T < S;
+    auto empty = [&](int k) { return may_be_empty && part_begin(k, T, S) == part_begin(k + 1, T, S); };
     // exponent base: the largest partial log-sum-exp of the row
     float m = -INFINITY;
     for (int k = k_first; k <= k_last; ++k) {
-        if (part_begin(k, T, S) == part_begin(k + 1, T, S)) continue;  // empty partition
+        if (empty(k)) continue;
         m = fmaxf(m, lse_part[(static_cast<int64_t>(b) + k) * rows + row]);
     }
     float4 acc[VEC];
@@ -51,7 +54,7 @@ __global__ void __launch_bounds__(256) combine_kernel(int batch, int q_len, int 
             for (int j = 0; j < 4; ++j) {
                 const int k = k4 + j;
                 wk[j] = 0.f;
-                if (k <= k_last && part_begin(k, T, S) != part_begin(k + 1, T, S)) {
+                if (k <= k_last && !empty(k)) {
                     const int64_t slot = static_cast<int64_t>(b) + k;
                     const float l = lse_part[slot * rows + row];
                     if (l != -INFINITY) {

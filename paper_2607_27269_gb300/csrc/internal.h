@@ -61,7 +61,8 @@ cudaError_t launch_out_proj(const mla_dims &d, int batch, int q_len, const float
 // C[phys(g, m), n] = sum_k A[phys(g, m), k] B_g(n, k) (bf16 result), with
 // phys(g, m) = (m / hpg) * blk + g * hpg + m % hpg.  A is fp32 or bf16 with
 // row stride lda; B_g(n, k) = B[g N K + n K + k] (K-major) or B[g K N + k N + n]
-// (N-major), bf16.  K and N are multiples of 8; A, B and C 16-byte aligned.
+// (N-major), bf16.  K and N are multiples of 8; A, B and C 16-byte aligned;
+// hpg <= 128 divides M.
 struct GroupGemm {
     int M, N, K, G;
     int hpg, blk;
