@@ -13,6 +13,8 @@ __global__ void __launch_bounds__(256) absorb_rope_kernel(int q_len, int H, int 
                                                          float base, const int32_t *__restrict__ kv_len,
                                                          const uint16_t *__restrict__ q_pe, uint16_t *q_abs)
 {
+    griddep_wait();
+    griddep_launch_dependents();
     __shared__ float cs[64], sn[64];
     const int bi = blockIdx.x;
     const int b = bi / q_len, i = bi % q_len;
@@ -58,10 +60,9 @@ cudaError_t launch_absorb(const mla_dims &d, int batch, int q_len, const void *q
     p.status = status;
     cudaError_t e = launch_group_gemm(p, st);
     if (e != cudaSuccess) return e;
-    absorb_rope_kernel<<<batch * q_len, 256, 0, st>>>(q_len, H, d.rank, d.d_rope, d.rope_style, d.rope_base, kv_len,
-                                                      static_cast<const uint16_t *>(q_pe),
-                                                      static_cast<uint16_t *>(q_abs));
-    return cudaGetLastError();
+    return launch_dependent(absorb_rope_kernel, dim3(batch * q_len), dim3(256), 0, st, 1, q_len, H, d.rank, d.d_rope,
+                            d.rope_style, d.rope_base, kv_len, static_cast<const uint16_t *>(q_pe),
+                            static_cast<uint16_t *>(q_abs));
 }
 
 }  // namespace gbmla

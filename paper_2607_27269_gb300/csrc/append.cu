@@ -16,6 +16,8 @@ __global__ void __launch_bounds__(128) cache_append_kernel(CacheView c, int rank
                                                           const int32_t *__restrict__ start_pos,
                                                           unsigned *status)
 {
+    griddep_wait();
+    griddep_launch_dependents();
     const int k = blockIdx.x, b = blockIdx.y;
     const int64_t pos = static_cast<int64_t>(start_pos[b]) + k;
     if (pos < 0 || pos >= c.capacity) {
@@ -62,10 +64,9 @@ cudaError_t launch_append(const mla_dims &d, const CacheView &c, int batch, int 
                           const void *kr_new, const int32_t *start_pos, unsigned *status, cudaStream_t st)
 {
     dim3 grid(n_new, batch);
-    cache_append_kernel<<<grid, 128, 0, st>>>(c, d.rank, d.d_rope, d.rope_style, d.rope_base, n_new,
-                                              static_cast<const uint16_t *>(c_new),
-                                              static_cast<const uint16_t *>(kr_new), start_pos, status);
-    return cudaGetLastError();
+    return launch_dependent(cache_append_kernel, grid, dim3(128), 0, st, 1, c, d.rank, d.d_rope, d.rope_style,
+                            d.rope_base, n_new, static_cast<const uint16_t *>(c_new),
+                            static_cast<const uint16_t *>(kr_new), start_pos, status);
 }
 
 }  // namespace gbmla

@@ -24,6 +24,8 @@ struct Smem {
 
 __global__ void __launch_bounds__(kThreads) attn_simt_kernel(AttnArgs a)
 {
+    griddep_wait();
+    griddep_launch_dependents();
     extern __shared__ __align__(16) unsigned char dyn[];
     __shared__ Smem sm;
     const int K = a.rank + a.d_rope;
@@ -208,7 +210,8 @@ cudaError_t launch_attn_simt(const AttnArgs &a, cudaStream_t st)
     if (e != cudaSuccess) return e;
     const int rows = a.q_len * a.num_heads;
     dim3 grid(a.num_splits, (rows + kRows - 1) / kRows);
-    attn_simt_kernel<<<grid, kThreads, smem, st>>>(a);
+    cudaError_t e0 = launch_dependent(attn_simt_kernel, grid, dim3(kThreads), smem, st, 1, a);
+    if (e0 != cudaSuccess) return e0;
     return cudaGetLastError();
 }
 

@@ -594,17 +594,6 @@ __global__ void __maxnreg__(128)
     const uint32_t rank_in_cluster = CL > 1 ? tc::cluster_ctarank() : 0;
     const uint64_t lim_ns = a.wait_ns;
 
-    if (part == 0 && group == 0) {
-        for (int bb = tid; bb < a.batch; bb += kThreads) {
-            const int kv = a.kv_len[bb];
-            if (kv < a.q_len || kv > a.max_kv) record_status(a.status, kStatusBounds);
-        }
-    }
-    const int64_t T = block_tile_sum(a.kv_len, a.batch, a.q_len, a.max_kv, red64);
-    const int64_t t_begin = T ? part_begin(part, T, a.num_splits) : 0;
-    const int64_t t_end = T ? part_begin(part + 1, T, a.num_splits) : 0;
-    const int n_items = static_cast<int>(t_end - t_begin);
-
     if (tid == 0) {
         for (int i = 0; i < kMaxSlots; ++i) {
             mbar_init(&bars.qk_full[i], 1);
@@ -648,6 +637,19 @@ __global__ void __maxnreg__(128)
     __syncthreads();
     if (CL > 1) tc::cluster_sync();  // peers may multicast into this CTA only after its barriers exist
     tc::fence_after_sync();
+    griddep_wait();  // the queries and the cache entries come from the previous launches
+    griddep_launch_dependents();
+
+    if (part == 0 && group == 0) {
+        for (int bb = tid; bb < a.batch; bb += kThreads) {
+            const int kv = a.kv_len[bb];
+            if (kv < a.q_len || kv > a.max_kv) record_status(a.status, kStatusBounds);
+        }
+    }
+    const int64_t T = block_tile_sum(a.kv_len, a.batch, a.q_len, a.max_kv, red64);
+    const int64_t t_begin = T ? part_begin(part, T, a.num_splits) : 0;
+    const int64_t t_end = T ? part_begin(part + 1, T, a.num_splits) : 0;
+    const int n_items = static_cast<int>(t_end - t_begin);
     const uint32_t tmem = ss.tmem_base;
     const uint32_t o_col0 = 2 * N;   // S^T buffers at columns [0, N) and [N, 2N)
     auto any_abort = [&]() {
@@ -1045,21 +1047,8 @@ cudaError_t launch_cfg(const AttnArgs &a, int groups, cudaStream_t st)
     t.lse_part = a.lse_part;
     t.status = a.status;
     t.wait_ns = kWaitLimitNs;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(groups, a.num_splits, 1);
-    cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    if (CL > 1) {
-        attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = CL;
-        attr[0].val.clusterDim.y = 1;
-        attr[0].val.clusterDim.z = 1;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
-    }
-    return cudaLaunchKernelEx(&cfg, attn_tc_kernel<N, CL>, t, mc, mr, mq);
+    return launch_dependent(attn_tc_kernel<N, CL>, dim3(groups, a.num_splits, 1), dim3(kThreads), smem, st, CL, t,
+                            mc, mr, mq);
 }
 
 }  // namespace

@@ -19,6 +19,8 @@ __global__ void __launch_bounds__(256) combine_kernel(int batch, int q_len, int 
                                                      const float *__restrict__ lse_part, float *o_lat,
                                                      float *lse_out)
 {
+    griddep_wait();
+    griddep_launch_dependents();
     __shared__ int64_t red[32];
     const int b = blockIdx.y;
     const int64_t T = block_tile_sum(kv_len, batch, q_len, max_kv, red);
@@ -99,9 +101,8 @@ cudaError_t launch_combine(int batch, int q_len, int num_heads, int rank, int ma
     const int rows = q_len * num_heads;
     dim3 grid((rows + rpb - 1) / rpb, batch);
     if (batch == 0 || rows == 0) return cudaSuccess;
-    combine_kernel<2><<<grid, 256, 0, st>>>(batch, q_len, num_heads, rank, max_kv, num_splits, kv_len, o_part,
-                                             lse_part, o_lat, lse);
-    return cudaGetLastError();
+    return launch_dependent(combine_kernel<2>, grid, dim3(256), 0, st, 1, batch, q_len, num_heads, rank, max_kv,
+                            num_splits, kv_len, o_part, lse_part, o_lat, lse);
 }
 
 }  // namespace gbmla

@@ -89,6 +89,8 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
     tc::fence_before_sync();
     __syncthreads();
     tc::fence_after_sync();
+    griddep_wait();  // the activations come from the previous launch
+    griddep_launch_dependents();
     const uint32_t tmem = tmem_base;
     auto bail = [&]() {
         record_status(p.status, kStatusTimeout);
@@ -289,8 +291,7 @@ cudaError_t launch_tc(const GroupGemm &p, cudaStream_t st)
     if (e != cudaSuccess) return e;
     const int rt = (128 / p.hpg) * p.hpg;
     dim3 grid((p.M + rt - 1) / rt, (p.N + BN - 1) / BN, p.G);
-    gemm_tc_kernel<BN, NMAJ, AF32><<<grid, kGemmThreads, smem, st>>>(p, ma, mb);
-    return cudaGetLastError();
+    return launch_dependent(gemm_tc_kernel<BN, NMAJ, AF32>, grid, dim3(kGemmThreads), smem, st, 1, p, ma, mb);
 }
 
 }  // namespace
