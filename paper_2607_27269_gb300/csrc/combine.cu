@@ -21,10 +21,10 @@ __global__ void __launch_bounds__(256) combine_kernel(int batch, int q_len, int 
 {
     griddep_wait();
     griddep_launch_dependents();
-    __shared__ int64_t red[32];
+    __shared__ int64_t red[64];
     const int b = blockIdx.y;
-    const int64_t T = block_tile_sum(kv_len, batch, q_len, max_kv, red);
-    const int64_t t0 = block_tile_sum(kv_len, b, q_len, max_kv, red);
+    int64_t T, t0;
+    block_tile_sums(kv_len, batch, b, q_len, max_kv, red, &T, &t0);
     const int64_t nb = seq_tiles(kv_len[b], q_len, max_kv);
     if (nb == 0 || T == 0) return;  // invalid length: recorded by the attention kernel
     const int k_first = part_of_tile(t0, T, S), k_last = part_of_tile(t0 + nb - 1, T, S);

@@ -155,6 +155,40 @@ __device__ __forceinline__ int64_t block_tile_sum(const int32_t *kv_len, int n, 
     return tot;
 }
 
+// One pass over the lengths: *total = all sequences' tiles, *before = the
+// tiles of sequences 0 .. b-1 (block-wide; every thread gets both).
+__device__ __forceinline__ void block_tile_sums(const int32_t *kv_len, int n, int b, int q_len, int capacity,
+                                                int64_t *red, int64_t *total, int64_t *before)
+{
+    int64_t acc = 0, pre = 0;
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+        const int64_t t = seq_tiles(kv_len[i], q_len, capacity);
+        acc += t;
+        if (i < b) pre += t;
+    }
+    for (int o = 16; o > 0; o >>= 1) {
+        acc += __shfl_xor_sync(0xffffffffu, acc, o);
+        pre += __shfl_xor_sync(0xffffffffu, pre, o);
+    }
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    __syncthreads();
+    if (lane == 0) {
+        red[2 * warp] = acc;
+        red[2 * warp + 1] = pre;
+    }
+    __syncthreads();
+    int64_t tot = 0, bef = 0;
+    const int nw = (blockDim.x + 31) >> 5;
+    for (int w = 0; w < nw; ++w) {
+        tot += red[2 * w];
+        bef += red[2 * w + 1];
+    }
+    __syncthreads();
+    *total = tot;
+    *before = bef;
+}
+
+
 // RoPE angle pos * theta_k reduced to [-pi, pi] in fp64 before the fp32
 // sincos, so that positions up to 2^31 keep fp32 accuracy.
 __device__ __forceinline__ void rope_cos_sin(int64_t pos, double theta, float *c, float *s)

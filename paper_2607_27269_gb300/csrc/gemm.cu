@@ -28,7 +28,7 @@ __device__ __forceinline__ int64_t phys_row(const GroupGemm &p, int g, int m)
 // of hpg rows, i.e. RT = R hpg <= 128 rows.  A bf16 A box lands directly in
 // the 128B-swizzled K-major layout the MMA reads; an fp32 A (o_lat) lands as
 // two 32-column boxes in a staging tile, which four warps convert to bf16.
-constexpr int kStages = 3;
+constexpr int kStages = 8;  // most ring stages; fewer when K is short or shared memory runs out
 constexpr int kGemmThreads = 192;  // warp 0 TMA, warp 1 MMA, warps 2..5 convert / epilogue
 
 struct __align__(8) GemmBars {
@@ -60,14 +60,15 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
     __shared__ int fail;
     unsigned char *smem = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                             ~static_cast<uintptr_t>(1023));
-    unsigned char *sa = smem;                            // kStages x A tile
-    unsigned char *sb = sa + kStages * kABytes;          // kStages x B tile
-    unsigned char *sr = sb + kStages * kBBytes;          // kStages x raw fp32 A (AF32)
+    const int nk = (p.K + 63) / 64;
+    const int NS = p.stages;                             // ring stages (<= kStages, <= nk)
+    unsigned char *sa = smem;                            // NS x A tile
+    unsigned char *sb = sa + NS * kABytes;               // NS x B tile
+    unsigned char *sr = sb + NS * kBBytes;               // NS x raw fp32 A (AF32)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int R = 128 / p.hpg, RT = R * p.hpg;           // row blocks and rows per tile
+    const int R = p.rblk, RT = R * p.hpg;                // row blocks and rows per tile (<= 128)
     const int mt = blockIdx.x, n0 = blockIdx.y * BN, g = blockIdx.z;
     const int m0 = mt * RT;
-    const int nk = (p.K + 63) / 64;
     const uint32_t a_bytes = static_cast<uint32_t>(RT) * 128;  // per 64-column (bf16) or 32-column (fp32) box
     const uint64_t lim = kWaitLimitNs;
 
@@ -104,7 +105,7 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
             tc::prefetch_tensormap(&map_b);
         }
         for (int c = 0; c < nk; ++c) {
-            const int s = c % kStages, round = c / kStages;
+            const int s = c % NS, round = c / NS;
             if (round >= 1 && !__all_sync(0xffffffffu, mbar_wait(smem_u32(&bars.empty[s]), (round - 1) & 1, lim))) {
                 if (lane == 0) bail();
                 break;
@@ -143,7 +144,7 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
         };
         bool ok = true;
         for (int c = 0; c < nk && ok; ++c) {
-            const int s = c % kStages, par = (c / kStages) & 1;
+            const int s = c % NS, par = (c / NS) & 1;
             ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&bars.full[s]), par, lim) &&
                                              (!AF32 || mbar_wait(smem_u32(&bars.conv_done[s]), par, lim)));
             if (!ok) break;
@@ -164,7 +165,7 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
             // ---- fp32 -> bf16: thread r converts tile row r (two 128-byte swizzled fp32 rows)
             const int r = tid - 64;
             for (int c = 0; c < nk; ++c) {
-                const int s = c % kStages, par = (c / kStages) & 1;
+                const int s = c % NS, par = (c / NS) & 1;
                 if (!__all_sync(0xffffffffu, mbar_wait(smem_u32(&bars.raw_full[s]), par, lim))) {
                     if (lane == 0) bail();
                     break;
@@ -248,14 +249,16 @@ cudaError_t launch_tc(const GroupGemm &p, cudaStream_t st)
     }
     if (p.hpg < 1 || p.hpg > 128 || p.M % p.hpg) return cudaErrorInvalidValue;
     const int es = AF32 ? 4 : 2;
+    // row blocks per tile: as many as fit 128 rows, but no more than there are
+    // (a short A box leaves the tile's other rows stale; their results are dropped)
+    const int rblk = (128 / p.hpg) < (p.M / p.hpg) ? (128 / p.hpg) : (p.M / p.hpg);
     CUtensorMap ma, mb;
     {   // A: (K, head in group, group, row block) with the row mapping's strides
         cuuint64_t dims[4] = {static_cast<cuuint64_t>(p.K), static_cast<cuuint64_t>(p.hpg),
                               static_cast<cuuint64_t>(p.G), static_cast<cuuint64_t>(p.M / p.hpg)};
         cuuint64_t strides[3] = {static_cast<cuuint64_t>(p.lda) * es, static_cast<cuuint64_t>(p.hpg) * p.lda * es,
                                  static_cast<cuuint64_t>(p.blk) * p.lda * es};
-        cuuint32_t box[4] = {AF32 ? 32u : 64u, static_cast<cuuint32_t>(p.hpg), 1u,
-                             static_cast<cuuint32_t>(128 / p.hpg)};
+        cuuint32_t box[4] = {AF32 ? 32u : 64u, static_cast<cuuint32_t>(p.hpg), 1u, static_cast<cuuint32_t>(rblk)};
         cuuint32_t es4[4] = {1, 1, 1, 1};
         CUresult r = g_encode_gemm(&ma, AF32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4,
                                    const_cast<void *>(p.A), dims, strides, box, es4, CU_TENSOR_MAP_INTERLEAVE_NONE,
@@ -284,14 +287,22 @@ cudaError_t launch_tc(const GroupGemm &p, cudaStream_t st)
                                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
     }
-    const size_t smem =
-        1024 + static_cast<size_t>(kStages) * (128 * 128 + BN * 128 + (AF32 ? 2 * 128 * 128 : 0));
+    const int nk = (p.K + 63) / 64;
+    const size_t per_stage = 128 * 128 + BN * 128 + (AF32 ? 2 * 128 * 128 : 0);
+    int ns = static_cast<int>((192 * 1024) / per_stage);
+    if (ns > kStages) ns = kStages;
+    if (ns > nk) ns = nk;
+    if (ns < 1) ns = 1;
+    GroupGemm q = p;
+    q.stages = ns;
+    q.rblk = rblk;
+    const size_t smem = 1024 + static_cast<size_t>(ns) * per_stage;
     cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, NMAJ, AF32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    const int rt = (128 / p.hpg) * p.hpg;
+    const int rt = rblk * p.hpg;
     dim3 grid((p.M + rt - 1) / rt, (p.N + BN - 1) / BN, p.G);
-    return launch_dependent(gemm_tc_kernel<BN, NMAJ, AF32>, grid, dim3(kGemmThreads), smem, st, 1, p, ma, mb);
+    return launch_dependent(gemm_tc_kernel<BN, NMAJ, AF32>, grid, dim3(kGemmThreads), smem, st, 1, q, ma, mb);
 }
 
 }  // namespace
