@@ -10,9 +10,10 @@
  * Conventions
  *   - bf16 inputs are read as their exact values (a bf16 is the top half of
  *     an IEEE binary32), all arithmetic is fp64, nothing is rounded in
- *     between.  The only rounding is orc_cache_append(), which must store
- *     bf16 into the cache like the GPU does; it rounds the exact fp64
- *     rotation once, to nearest-even.
+ *     between.  The only roundings are the cache writes of
+ *     orc_cache_append() and orc_project_append(), which must store bf16
+ *     into the cache like the GPU does; each rounds the exact fp64 value
+ *     (rotation, projection) once, to nearest-even.
  *   - The attention is computed in its plain, NON-absorbed form: every cached
  *     latent c_j is up-projected to an explicit key k_j^nope = W_UK[g] c_j and
  *     value v_j = W_UV[g] c_j (Sec. 3.2, Eq. 5), and the scaled causal softmax
@@ -367,4 +368,79 @@ int orc_mla_decode(const orc_dims *d, const orc_cache *c, int batch, int q_len,
         }
     }
     return ORC_OK;
+}
+
+/* Projection of new hidden states into the cache and the queries, ahead of
+ * the decode step (Sec. 3.2: the latent c_j = W^DKV h_j and a positional key
+ * k^PE_j that is kept on the rotary path; Sec. 3.1 Eq. 1: q_{t,i} = W^Q_i h_t).
+ * Readings: k^PE_j = R_j (W^KR h_j), one positional key shared by every head;
+ * the converted query of head i is [q_nope (d_nope) ; q_pe (d_rope)], the
+ * first part on the non-positional path and the second on the rotary path
+ * (Sec. 3.3 routing).  Entry k of sequence b sits at position
+ * start_pos[b] + k.  Every projection is an exact fp64 dot product of the
+ * bf16 values; the cache receives the latent and the rotated positional key
+ * each rounded once to bf16 (the rotation is applied to the exact fp64
+ * projection), the queries are returned unrounded and unrotated.
+ *   h      [batch, n_new, D] bf16, D = d->hidden (> 0)
+ *   w_dkv  [rank, D], w_kr [d_rope, D], w_q [H (d_nope + d_rope), D] bf16
+ *          (w_q may be NULL: no query projection)
+ *   q_nope [batch, n_new, H, d_nope], q_pe [batch, n_new, H, d_rope] fp64 out
+ *          (ignored when w_q is NULL) */
+int orc_project_append(const orc_dims *d, const orc_cache *c, int batch, int n_new, const uint16_t *h,
+                       const uint16_t *w_dkv, const uint16_t *w_kr, const uint16_t *w_q,
+                       const int32_t *start_pos, double *q_nope, double *q_pe)
+{
+    if (check_dims(d) || batch < 0 || n_new < 0 || d->hidden <= 0) return ORC_BAD_ARG;
+    const int D = d->hidden, r = d->rank, dr = d->d_rope, dn = d->d_nope, H = d->num_heads;
+    const int dq = dn + dr;
+    /* positions and pages first, so that a bad entry leaves the cache untouched */
+    for (int b = 0; b < batch; ++b)
+        for (int k = 0; k < n_new; ++k) {
+            int64_t co, ro;
+            int err = tok_offsets(c, b, (int64_t)start_pos[b] + k, &co, &ro);
+            if (err) return err;
+        }
+    const int64_t rows = (int64_t)batch * n_new;
+    int err = ORC_OK;
+#pragma omp parallel for schedule(static)
+    for (int64_t row = 0; row < rows; ++row) {
+        const int b = (int)(row / (n_new > 0 ? n_new : 1)), k = (int)(row % (n_new > 0 ? n_new : 1));
+        const int64_t pos = (int64_t)start_pos[b] + k;
+        int64_t co, ro;
+        tok_offsets(c, b, pos, &co, &ro);
+        double *x = (double *)malloc(sizeof(double) * (size_t)(D + dr + 1));
+        if (!x) {
+#pragma omp critical
+            err = ORC_NO_MEMORY;
+            continue;
+        }
+        double *kr = x + D;
+        for (int e = 0; e < D; ++e) x[e] = orc_bf16_value(h[row * D + e]);
+        for (int e = 0; e < r; ++e) {  /* c = W^DKV h */
+            double acc = 0.0;
+            for (int t = 0; t < D; ++t) acc += orc_bf16_value(w_dkv[(int64_t)e * D + t]) * x[t];
+            c->c_kv[co + e] = orc_bf16_round(acc);
+        }
+        for (int e = 0; e < dr; ++e) {  /* k^PE = R_pos W^KR h */
+            double acc = 0.0;
+            for (int t = 0; t < D; ++t) acc += orc_bf16_value(w_kr[(int64_t)e * D + t]) * x[t];
+            kr[e] = acc;
+        }
+        orc_rope(kr, kr, dr, pos, d->rope_base, d->rope_style);
+        for (int e = 0; e < dr; ++e) c->k_rope[ro + e] = orc_bf16_round(kr[e]);
+        if (w_q) {  /* q_i = W^Q_i h, split into the two paths */
+            for (int hd = 0; hd < H; ++hd)
+                for (int e = 0; e < dq; ++e) {
+                    const uint16_t *w = w_q + ((int64_t)hd * dq + e) * D;
+                    double acc = 0.0;
+                    for (int t = 0; t < D; ++t) acc += orc_bf16_value(w[t]) * x[t];
+                    if (e < dn)
+                        q_nope[(row * H + hd) * dn + e] = acc;
+                    else
+                        q_pe[(row * H + hd) * dr + (e - dn)] = acc;
+                }
+        }
+        free(x);
+    }
+    return err;
 }

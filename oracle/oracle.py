@@ -115,6 +115,9 @@ def configure(lib):
     lib.orc_absorb_q.restype = ctypes.c_int
     lib.orc_absorb_q.argtypes = [ctypes.POINTER(_Dims), ctypes.c_int, ctypes.c_int, vp, vp, vp, vp,
                                  vp, vp]
+    lib.orc_project_append.restype = ctypes.c_int
+    lib.orc_project_append.argtypes = [ctypes.POINTER(_Dims), ctypes.POINTER(_Cache), ctypes.c_int, ctypes.c_int,
+                                       vp, vp, vp, vp, vp, vp, vp]
     lib.orc_mla_decode.restype = ctypes.c_int
     lib.orc_mla_decode.argtypes = [ctypes.POINTER(_Dims), ctypes.POINTER(_Cache), ctypes.c_int,
                                    ctypes.c_int, vp, vp, vp, vp, vp, vp, vp, ctypes.c_int,
@@ -219,6 +222,24 @@ def cache_append(dims: Dims, cache: Cache, c_new: np.ndarray, kr_new: np.ndarray
     d, c = dims._c(), cache._c()
     _check(_load().orc_cache_append(ctypes.byref(d), ctypes.byref(c), batch, n_new, c_new.ctypes.data,
                                     kr_new.ctypes.data, start_pos.ctypes.data), "cache_append")
+
+
+def project_append(dims: Dims, cache: Cache, h: np.ndarray, w_dkv: np.ndarray, w_kr: np.ndarray,
+                   w_q: Optional[np.ndarray], start_pos):
+    """Project hidden states h [B, n, D] into the cache and the queries
+    (Sec. 3.2 latent c = W^DKV h with the rotated positional key R_pos W^KR h;
+    Sec. 3.1 Eq. 1 q_i = W^Q_i h).  Writes the cache in place; returns
+    (q_nope, q_pe) fp64 (None without ``w_q``)."""
+    h, w_dkv, w_kr, start_pos = _u16(h), _u16(w_dkv), _u16(w_kr), _i32(start_pos)
+    w_q = None if w_q is None else _u16(w_q)
+    batch, n_new = h.shape[0], h.shape[1]
+    q_nope = np.zeros((batch, n_new, dims.num_heads, dims.d_nope)) if w_q is not None else None
+    q_pe = np.zeros((batch, n_new, dims.num_heads, dims.d_rope)) if w_q is not None else None
+    d, c = dims._c(), cache._c()
+    _check(_load().orc_project_append(ctypes.byref(d), ctypes.byref(c), batch, n_new, h.ctypes.data,
+                                      w_dkv.ctypes.data, w_kr.ctypes.data, _ptr(w_q), start_pos.ctypes.data,
+                                      _ptr(q_nope), _ptr(q_pe)), "project_append")
+    return q_nope, q_pe
 
 
 def absorb_q(dims: Dims, q_nope: np.ndarray, q_pe: np.ndarray, kv_len, w_uk: np.ndarray):

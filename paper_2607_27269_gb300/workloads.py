@@ -22,6 +22,12 @@ Recipe (one ``torch.Generator('cpu')`` seeded with ``seed``, drawn in this order
   6. the entries appended this step, c_new [B, q, r], kr_new [B, q, d_rope]
      ~ N(0, 1) (kr_new not yet rotated).
 Every tensor is drawn in fp32 and rounded to bf16.
+
+Inputs of the projection that precedes the step (``projection``) come from a
+second generator seeded with ``seed + 7919``, drawn in this order: hidden
+states h [B, q, D] ~ N(0, 1); W^DKV [r, D], W^KR [d_rope, D] and
+W^Q [H (d_nope + d_rope), D] ~ N(0, 1/sqrt(D)), so that the projected latents
+and keys have unit variance like the cache above.
 """
 from __future__ import annotations
 
@@ -183,3 +189,29 @@ def small(name: str, seed: int = 0) -> Workload:
     if s.kv_lo != s.kv_hi:
         return make(s, seed, batch=3, kv_range=(300, 1100))
     return make(s, seed, batch=3, kv_range=(517, 517))
+
+
+@dataclass
+class Projection:
+    """Hidden states and stacked projection weights of the step's new tokens."""
+    hidden: int                   # D
+    h: torch.Tensor               # bf16 [B, q, D]
+    w_dkv: torch.Tensor           # bf16 [r, D]
+    w_kr: torch.Tensor            # bf16 [d_rope, D]
+    w_q: torch.Tensor             # bf16 [H (d_nope + d_rope), D]
+
+
+def projection(w: Workload, seed: int = 0, hidden: Optional[int] = None) -> Projection:
+    """Projection inputs for workload ``w``'s new tokens; D = the shape's
+    hidden width (256 for a shape without one) unless ``hidden`` is given."""
+    s = w.shape
+    D = hidden if hidden is not None else (s.hidden if s.hidden > 0 else 256)
+    gen = torch.Generator(device="cpu")
+    gen.manual_seed(seed + 7919)
+    B, q = w.c_new.shape[0], w.c_new.shape[1]
+    std = 1.0 / math.sqrt(D)
+    h = _randn(gen, (B, q, D))
+    w_dkv = _randn(gen, (s.rank, D), std)
+    w_kr = _randn(gen, (s.d_rope, D), std)
+    w_q = _randn(gen, (s.num_heads * (s.d_nope + s.d_rope), D), std)
+    return Projection(D, h, w_dkv, w_kr, w_q)

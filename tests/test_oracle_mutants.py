@@ -29,6 +29,12 @@ MUTANTS = {
     "append_position_shift": ("int64_t pos = (int64_t)start_pos[b] + k, co, ro;",
                               "int64_t pos = (int64_t)start_pos[b] + k + 1, co, ro;"),
     "page_slot": ("slot = t % c->page_size;", "slot = (t + 1) % c->page_size;"),
+    "latent_projection_transposed": ("acc += orc_bf16_value(w_dkv[(int64_t)e * D + t]) * x[t];",
+                                     "acc += orc_bf16_value(w_dkv[((int64_t)t * r + e) % ((int64_t)r * D)]) * x[t];"),
+    "projected_key_unrotated": ("orc_rope(kr, kr, dr, pos, d->rope_base, d->rope_style);\n        for (int e = 0; e < dr; ++e) c->k_rope",
+                                "orc_rope(kr, kr, dr, 0, d->rope_base, d->rope_style);\n        for (int e = 0; e < dr; ++e) c->k_rope"),
+    "query_rows_head_interleaved": ("const uint16_t *w = w_q + ((int64_t)hd * dq + e) * D;",
+                                    "const uint16_t *w = w_q + ((int64_t)e * H + hd) * D;"),
     "output_projection_index": ("acc += orc_bf16_value(w[h * dv + e]) * o[(row0 + h) * dv + e];",
                                 "acc += orc_bf16_value(w[e * H + h]) * o[(row0 + h) * dv + e];"),
 }

@@ -411,3 +411,108 @@ def test_append_position_zero_is_a_copy_and_errors():
     cp.block_table[0, 1] = -1
     with pytest.raises(orc.OracleError, match="bad page"):
         orc.cache_append(dims_of(wp), cp, bits(wp.c_new), bits(wp.kr_new), wp.start_pos.numpy())
+
+
+# ---------------------------------------------------------------- projection + append (Sec. 3.2, Eq. 1)
+
+def _proj_case(paged=False, batch=3, q_len=2, kv=(3, 9), D=24, seed=5):
+    w = _tiny(batch=batch, q_len=q_len, kv=kv, paged=paged, seed=seed)
+    p = wl.projection(w, seed=seed, hidden=D)
+    dims = dataclasses.replace(dims_of(w), hidden=D)
+    return w, p, dims
+
+
+def _within_half_ulp(got_bits, exact):
+    got = bf16_to_f64(got_bits)
+    ulp = 2.0 ** (np.floor(np.log2(np.maximum(np.abs(exact), 1e-30))) - 7)
+    return np.all(np.abs(got - exact) <= ulp / 2 + 1e-15)
+
+
+def test_projection_of_unit_vectors_selects_weight_columns():
+    """h = e_k gives column k of every weight: the latent and the queries
+    exactly, the positional key exactly at position 0 and rotated elsewhere."""
+    w, p, dims = _proj_case(batch=2, q_len=3, kv=(3, 6))
+    s = w.shape
+    D = p.hidden
+    ks = [[0, 5, D - 1], [7, 11, 2]]
+    h = np.zeros((2, 3, D), dtype=np.uint16)
+    for b in range(2):
+        for i in range(3):
+            h[b, i, ks[b][i]] = 0x3F80                                   # bf16 1.0
+    start = np.array([0, int(w.start_pos[1])], dtype=np.int32)
+    cache = oracle_cache(w)
+    q_nope, q_pe = orc.project_append(dims, cache, h, bits(p.w_dkv), bits(p.w_kr), bits(p.w_q), start)
+    wd, wk, wq = bits(p.w_dkv), bits(p.w_kr), bf16_to_f64(bits(p.w_q))
+    dq = s.d_nope + s.d_rope
+    for b in range(2):
+        for i in range(3):
+            k, pos = ks[b][i], int(start[b]) + i
+            assert np.array_equal(cache.c_kv[b, pos], wd[:, k])
+            if pos == 0:
+                assert np.array_equal(cache.k_rope[b, pos], wk[:, k])   # R_0 = I
+            exact = rope_complex(bf16_to_f64(wk[:, k]), pos, s.rope_base, s.rope_style)
+            assert _within_half_ulp(cache.k_rope[b, pos], exact)
+            col = wq[:, k].reshape(s.num_heads, dq)
+            assert np.array_equal(q_nope[b, i], col[:, :s.d_nope])
+            assert np.array_equal(q_pe[b, i], col[:, s.d_nope:])
+
+
+@pytest.mark.parametrize("style", [0, 1])
+def test_projection_matches_matmul_and_rounds_once(style):
+    """Random inputs: the cache rows are the numpy fp64 products rounded once
+    (the positional key rotated first, by the complex form), the queries are
+    the products themselves."""
+    w, p, dims = _proj_case(seed=6)
+    w = dataclasses.replace(w, shape=dataclasses.replace(w.shape, rope_style=style))
+    dims = dataclasses.replace(dims, rope_style=style)
+    s = w.shape
+    before_c, before_r = bits(w.c_kv), bits(w.k_rope)
+    cache = oracle_cache(w)
+    q_nope, q_pe = orc.project_append(dims, cache, bits(p.h), bits(p.w_dkv), bits(p.w_kr), bits(p.w_q),
+                                      w.start_pos.numpy())
+    h = bf16_to_f64(bits(p.h))
+    c = h @ bf16_to_f64(bits(p.w_dkv)).T
+    kr = h @ bf16_to_f64(bits(p.w_kr)).T
+    q = (h @ bf16_to_f64(bits(p.w_q)).T).reshape(*h.shape[:2], s.num_heads, s.d_nope + s.d_rope)
+    np.testing.assert_allclose(q_nope, q[..., :s.d_nope], rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(q_pe, q[..., s.d_nope:], rtol=1e-12, atol=1e-12)
+    for b in range(s.batch):
+        sp = int(w.start_pos[b])
+        for t in range(w.capacity):
+            if sp <= t < sp + s.q_len:
+                assert _within_half_ulp(cache.c_kv[b, t], c[b, t - sp])
+                assert _within_half_ulp(cache.k_rope[b, t],
+                                        rope_complex(kr[b, t - sp], t, s.rope_base, style))
+            else:
+                assert np.array_equal(cache.c_kv[b, t], before_c[b, t])
+                assert np.array_equal(cache.k_rope[b, t], before_r[b, t])
+
+
+def test_projection_paged_equals_contiguous_and_errors():
+    """The paged cache receives the same rows at block_table[b][t // P],
+    slot t % P; a position past the capacity or a bad page is an error that
+    leaves the cache untouched."""
+    wp, p, dims = _proj_case(paged=True, seed=8)
+    cp = oracle_cache(wp)
+    orc.project_append(dims, cp, bits(p.h), bits(p.w_dkv), bits(p.w_kr), None, wp.start_pos.numpy())
+    s = wp.shape
+    cap = int(wp.kv_len.max())
+    cc = np.zeros((s.batch, cap, s.rank), dtype=np.uint16)
+    rc = np.zeros((s.batch, cap, s.d_rope), dtype=np.uint16)
+    ccache = orc.Cache(c_kv=cc, k_rope=rc, c_tok_stride=s.rank, r_tok_stride=s.d_rope,
+                       c_blk_stride=cap * s.rank, r_blk_stride=cap * s.d_rope, capacity=cap)
+    orc.project_append(dims, ccache, bits(p.h), bits(p.w_dkv), bits(p.w_kr), None, wp.start_pos.numpy())
+    for b in range(s.batch):
+        for t in range(int(wp.start_pos[b]), int(wp.kv_len[b])):
+            blk, slot = cp.block_table[b, t // s.page_size], t % s.page_size
+            assert np.array_equal(cp.c_kv[blk, slot], cc[b, t])
+            assert np.array_equal(cp.k_rope[blk, slot], rc[b, t])
+    bad = oracle_cache(wp)
+    snapshot = bad.c_kv.copy()
+    bad.block_table[s.batch - 1, (int(wp.kv_len[-1]) - 1) // s.page_size] = -1
+    with pytest.raises(orc.OracleError, match="bad page"):
+        orc.project_append(dims, bad, bits(p.h), bits(p.w_dkv), bits(p.w_kr), None, wp.start_pos.numpy())
+    assert np.array_equal(bad.c_kv, snapshot)
+    with pytest.raises(orc.OracleError, match="bad position"):
+        orc.project_append(dims, oracle_cache(wp), bits(p.h), bits(p.w_dkv), bits(p.w_kr), None,
+                           np.full(s.batch, wp.capacity, dtype=np.int32))
