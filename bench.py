@@ -248,6 +248,8 @@ def run_ours(args, rank, world, local):
         torch.cuda.synchronize(dev)
         attn_ms = [a.elapsed_time(b) / n_attn for a, b in attn_ms]
 
+        proj = measure_projection(args, w, dws, stream, dev, l2, peaks=load_peaks())
+
         # ---- end to end through the public API with host buffers
         host_in = {k: getattr(w, k).pin_memory() for k in ("q_nope", "q_pe", "c_new", "kr_new", "kv_len", "start_pos")}
         out_dev = steps[0].out if steps[0].out is not None else steps[0].o
@@ -322,8 +324,74 @@ def run_ours(args, rank, world, local):
                 "us_per_step": round(max_e2e / args.steps * 1e3, 3),
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": launches_per_step * args.steps,
+        "project_append": proj,
     }
     return line, w
+
+
+def measure_projection(args, w, dws, stream, dev, l2, peaks):
+    """The projection that precedes the step (mla_project_append) timed alone:
+    a CUDA graph of back-to-back launches over enough weight replicas that
+    the weights streamed between two reuses exceed 2x L2.  Reported beside
+    the step (it is not part of the step's bytes)."""
+    import torch
+    from paper_2607_27269_gb300 import abi
+    from paper_2607_27269_gb300 import workloads as wl
+
+    s = w.shape
+    p = wl.projection(w, seed=args.seed)
+    D = p.hidden
+    B, n = w.c_new.shape[0], w.c_new.shape[1]
+    M = B * n
+    nq = s.num_heads * (s.d_nope + s.d_rope)
+    weight_bytes = (s.rank + s.d_rope + nq) * D * 2
+    io_bytes = M * D * 2 + M * (s.rank + s.d_rope + nq) * 2
+    flops = 2.0 * M * D * (s.rank + s.d_rope + nq)
+    reps = max(2, math.ceil(2 * l2 / weight_bytes) + 1)
+    dims = abi.Dims(s.num_heads, s.num_kv_groups, s.d_nope, s.d_rope, s.d_v, s.rank, D, s.sm_scale, s.rope_style,
+                    s.rope_base)
+    h = p.h.to(dev)
+    ws = [(p.w_dkv.to(dev), p.w_kr.to(dev), p.w_q.to(dev)) for _ in range(reps)]
+    q_nope = torch.empty(B, n, s.num_heads, s.d_nope, dtype=torch.bfloat16, device=dev)
+    q_pe = torch.empty(B, n, s.num_heads, s.d_rope, dtype=torch.bfloat16, device=dev)
+    n_launch = max(reps, 32)
+
+    def launch(i):
+        d = dws[i % len(dws)]
+        w_dkv, w_kr, w_q = ws[i % reps]
+        abi.project_append(dims, d.cache, h, w_dkv, w_kr, w_q, d.start_pos, q_nope, q_pe, stream)
+
+    for i in range(3):
+        launch(i)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for i in range(n_launch):
+            launch(i)
+    g.replay()
+    torch.cuda.synchronize(dev)
+    times = []
+    for _ in range(5):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        g.replay()
+        b.record(stream)
+        times.append((a, b))
+    torch.cuda.synchronize(dev)
+    code = abi.check_status(stream)
+    if code != abi.MLA_OK:
+        raise RuntimeError(f"device status after the projection: {abi.status_name(code)}")
+    us = sum(a.elapsed_time(b) for a, b in times) / len(times) / n_launch * 1e3
+    gbs = (weight_bytes + io_bytes) / (us * 1e-6) / 1e9
+    tflops = flops / (us * 1e-6) / 1e12
+    # the bound is whichever roofline time is longer at the measured peaks
+    t_hbm = (weight_bytes + io_bytes) / (peaks["hbm_gbs"] * 1e9)
+    t_tc = flops / (peaks["bf16_tflops"] * 1e12)
+    bound = "tensor" if t_tc > t_hbm else "hbm"
+    frac = (tflops / peaks["bf16_tflops"]) if bound == "tensor" else (gbs / peaks["hbm_gbs"])
+    return {"kernel": "mla_project_append", "us_per_launch": round(us, 3), "rows": M, "hidden": D,
+            "columns": s.rank + s.d_rope + nq, "bytes_per_launch": weight_bytes + io_bytes,
+            "flops_per_launch": flops, "achieved_gbs": round(gbs, 1), "achieved_tflops": round(tflops, 2),
+            "bound": bound, "frac": round(frac, 4), "weight_replicas": reps, "peak_source": peaks["source"]}
 
 
 # DRAM bytes (read + write) per attention launch from one ncu capture of the

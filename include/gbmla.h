@@ -5,6 +5,9 @@
  * The step a draft runs at every proposal (q_len = 1) and every catch-up
  * chunk (q_len = gamma + 1) is
  *
+ *   mla_project_append (optional, replaces mla_cache_append when the caller
+ *                      holds hidden states) project h into the latent and
+ *                      positional caches and the queries     (Sec. 3.2, Eq. 1)
  *   mla_cache_append   write this step's latent rows c_j and RoPE-rotated
  *                      positional keys k_j^PE into the cache    (Sec. 3.2, Sec. 3.1)
  *   mla_absorb_q       q_lat = W_UK[g]^T q_nope, RoPE the positional query
@@ -132,6 +135,30 @@ mla_status mla_workspace_size(const mla_dims *dims, int32_t batch, int32_t q_len
  * skipped and recorded as MLA_ERR_DEVICE_BOUNDS.  batch or n_new == 0: no-op. */
 mla_status mla_cache_append(const mla_dims *dims, const mla_cache *cache, int32_t batch, int32_t n_new,
                             const void *c_new, const void *kr_new, const int32_t *start_pos, void *stream);
+
+/* Projection of this step's hidden states into the cache and the queries,
+ * the work that precedes mla_cache_append / mla_absorb_q, as one launch
+ * (Sec. 3.2: latent c_j = W^DKV h_j and positional key k^PE_j = R_j W^KR h_j,
+ * one key shared by all heads; Sec. 3.1 Eq. 1: q_{t,i} = W^Q_i h_t, whose
+ * first d_nope entries take the non-positional path and the last d_rope the
+ * rotary path).  For every sequence b and entry k < n_new, position
+ * p = start_pos[b] + k and x = h[b, k, :]:
+ *   c_kv row (b, p)     <- bf16(W_DKV x)          (fp32 accumulation, one RNE rounding)
+ *   k_rope row (b, p)   <- bf16(R_p (W_KR x))     (the fp32 sum rotated in fp32, one rounding)
+ *   q_nope[b, k, h, :]  <- bf16((W_Q x)[h dq .. h dq + d_nope))
+ *   q_pe[b, k, h, :]    <- bf16((W_Q x)[h dq + d_nope .. (h + 1) dq))   (not rotated)
+ * with dq = d_nope + d_rope.  h [batch, n_new, hidden] bf16 with
+ * hidden = dims->hidden > 0 and a multiple of 8; W_DKV [rank, hidden],
+ * W_KR [d_rope, hidden], W_Q [H dq, hidden] bf16; q_nope [batch, n_new, H,
+ * d_nope] and q_pe [batch, n_new, H, d_rope] bf16; start_pos [batch] int32
+ * device; every bf16 pointer 16-byte aligned.  w_q == NULL skips the queries
+ * (q_nope and q_pe may then be NULL).  A position outside [0, capacity) or a
+ * page outside [0, num_pages) skips that entry's cache rows and is recorded
+ * as MLA_ERR_DEVICE_BOUNDS; its queries are still written.  batch or
+ * n_new == 0: no-op. */
+mla_status mla_project_append(const mla_dims *dims, const mla_cache *cache, int32_t batch, int32_t n_new,
+                              const void *h, const void *w_dkv, const void *w_kr, const void *w_q,
+                              const int32_t *start_pos, void *q_nope, void *q_pe, void *stream);
 
 /* Query absorption (Sec. 1; Eq. 5): for each (b, i, h)
  *   q_abs[b, i, h, 0:r]        = sum_d q_nope[b, i, h, d] * W_UK[g(h), d, :]

@@ -19,7 +19,7 @@ from . import build as _build
 
 MLA_OK, MLA_ERR_INVALID_ARG, MLA_ERR_UNSUPPORTED, MLA_ERR_CUDA, MLA_ERR_DEVICE_BOUNDS, MLA_ERR_DEVICE_TIMEOUT = range(6)
 SPLIT_TILE = 128
-EXPORTS = ("mla_workspace_size", "mla_cache_append", "mla_absorb_q", "mla_decode_attn", "mla_combine",
+EXPORTS = ("mla_workspace_size", "mla_cache_append", "mla_project_append", "mla_absorb_q", "mla_decode_attn", "mla_combine",
            "mla_out_proj", "mla_check_status", "mla_selftest_wait_timeout", "mla_decode_attn_noalloc",
            "mla_status_str", "mla_last_error")
 
@@ -69,6 +69,7 @@ def lib(auto_build: bool = True):
             L.mla_status_str.argtypes = [ctypes.c_int]
             L.mla_workspace_size.argtypes = [P(MlaDims), i32, i32, i32, i32, P(sz), P(sz), P(i32)]
             L.mla_cache_append.argtypes = [P(MlaDims), P(MlaCache), i32, i32, vp, vp, vp, vp]
+            L.mla_project_append.argtypes = [P(MlaDims), P(MlaCache), i32, i32, vp, vp, vp, vp, vp, vp, vp, vp]
             L.mla_absorb_q.argtypes = [P(MlaDims), i32, i32, vp, vp, vp, vp, vp, vp]
             L.mla_decode_attn.argtypes = [P(MlaDims), P(MlaCache), i32, i32, vp, i32, vp, i32, vp, vp, vp]
             L.mla_combine.argtypes = [P(MlaDims), i32, i32, i32, vp, i32, vp, vp, vp, vp, vp]
@@ -168,6 +169,17 @@ def cache_append(dims: Dims, cache: Cache, c_new: torch.Tensor, kr_new: torch.Te
                                                       _p(c_new), _p(kr_new), _p(start_pos), _stream(stream)))
 
 
+def project_append(dims: Dims, cache: Cache, h: torch.Tensor, w_dkv: torch.Tensor, w_kr: torch.Tensor,
+                   w_q: Optional[torch.Tensor], start_pos: torch.Tensor, q_nope: Optional[torch.Tensor] = None,
+                   q_pe: Optional[torch.Tensor] = None, stream=None):
+    """h [B, n, hidden] -> cache rows at start_pos + k and, with ``w_q``, the
+    query parts q_nope [B, n, H, d_nope] / q_pe [B, n, H, d_rope]."""
+    batch, n_new = h.shape[0], h.shape[1]
+    _check("mla_project_append", lib().mla_project_append(ctypes.byref(dims.c()), ctypes.byref(cache.c()), batch,
+                                                          n_new, _p(h), _p(w_dkv), _p(w_kr), _p(w_q),
+                                                          _p(start_pos), _p(q_nope), _p(q_pe), _stream(stream)))
+
+
 def absorb_q(dims: Dims, q_nope: torch.Tensor, q_pe: torch.Tensor, kv_len: torch.Tensor, w_uk: torch.Tensor,
              q_abs: torch.Tensor, stream=None):
     batch, q_len = q_nope.shape[0], q_nope.shape[1]
@@ -219,7 +231,8 @@ def selftest_wait_timeout(limit_ns: int, stream=None):
 class DecodeStep:
     """One decode step of an MLA layer through the five entry points, with
     every intermediate buffer allocated once (by PyTorch) up front:
-    append -> absorb -> split-KV attention -> combine -> up/out projection."""
+    append -> absorb -> split-KV attention -> combine -> up/out projection
+    (or, through ``from_hidden``, projection -> absorb -> ...)."""
 
     def __init__(self, dims: Dims, cache: Cache, batch: int, q_len: int, max_kv_len: int, num_splits: int = 0,
                  device=None):
@@ -251,6 +264,18 @@ class DecodeStep:
                 self.num_splits, stream)
         out_proj(d, self.o_lat, w_uv, w_o if d.hidden else None, self.o, self.out if d.hidden else None, stream)
         return self.out if (d.hidden and w_o is not None) else self.o
+
+    def from_hidden(self, h, w_dkv, w_kr, w_q, start_pos, kv_len, w_uk, w_uv, w_o=None, stream=None):
+        """The step fed by hidden states h [B, q_len, hidden]: the projection
+        writes the cache rows and the queries (kept in ``self.q_nope`` /
+        ``self.q_pe``), then absorption, attention, combine and projections."""
+        d = self.dims
+        if getattr(self, "q_nope", None) is None:
+            dev = h.device
+            self.q_nope = torch.empty(self.batch, self.q_len, d.num_heads, d.d_nope, dtype=torch.bfloat16, device=dev)
+            self.q_pe = torch.empty(self.batch, self.q_len, d.num_heads, d.d_rope, dtype=torch.bfloat16, device=dev)
+        project_append(d, self.cache, h, w_dkv, w_kr, w_q, start_pos, self.q_nope, self.q_pe, stream)
+        return self(self.q_nope, self.q_pe, kv_len, w_uk, w_uv, w_o, stream=stream)
 
 
 @dataclass

@@ -10,7 +10,7 @@ namespace {
 // One block per (b, i): angles of position kv_len[b] - q_len + i are shared
 // by all heads.
 __global__ void __launch_bounds__(256) absorb_rope_kernel(int q_len, int H, int rank, int d_rope, int style,
-                                                         float base, const int32_t *__restrict__ kv_len,
+                                                         const RopeTurns turns, const int32_t *__restrict__ kv_len,
                                                          const uint16_t *__restrict__ q_pe, uint16_t *q_abs)
 {
     griddep_wait();
@@ -20,7 +20,7 @@ __global__ void __launch_bounds__(256) absorb_rope_kernel(int q_len, int H, int 
     const int b = bi / q_len, i = bi % q_len;
     const int half = d_rope / 2;
     const int64_t pos = static_cast<int64_t>(kv_len[b]) - q_len + i;
-    for (int e = threadIdx.x; e < half; e += blockDim.x) rope_cos_sin(pos, rope_theta(e, d_rope, base), &cs[e], &sn[e]);
+    for (int e = threadIdx.x; e < half; e += blockDim.x) rope_cos_sin(pos, turns.f[e], &cs[e], &sn[e]);
     __syncthreads();
     const int ld = rank + d_rope;
     for (int t = threadIdx.x; t < H * half; t += blockDim.x) {
@@ -61,7 +61,7 @@ cudaError_t launch_absorb(const mla_dims &d, int batch, int q_len, const void *q
     cudaError_t e = launch_group_gemm(p, st);
     if (e != cudaSuccess) return e;
     return launch_dependent(absorb_rope_kernel, dim3(batch * q_len), dim3(256), 0, st, 1, q_len, H, d.rank, d.d_rope,
-                            d.rope_style, d.rope_base, kv_len, static_cast<const uint16_t *>(q_pe),
+                            d.rope_style, rope_turns(d.d_rope, d.rope_base), kv_len, static_cast<const uint16_t *>(q_pe),
                             static_cast<uint16_t *>(q_abs));
 }
 

@@ -225,6 +225,28 @@ mla_status mla_cache_append(const mla_dims *dims, const mla_cache *cache, int32_
                                    static_cast<cudaStream_t>(stream)));
 }
 
+mla_status mla_project_append(const mla_dims *dims, const mla_cache *cache, int32_t batch, int32_t n_new,
+                              const void *h, const void *w_dkv, const void *w_kr, const void *w_q,
+                              const int32_t *start_pos, void *q_nope, void *q_pe, void *stream)
+{
+    mla_status s = check_dims(dims);
+    if (s != MLA_OK) return s;
+    CacheView v;
+    if ((s = check_cache(dims, cache, &v)) != MLA_OK) return s;
+    if (batch < 0 || n_new < 0 || batch > 65535 || n_new > 65535) return MLA_ERR_INVALID_ARG;
+    if (dims->hidden <= 0 || dims->hidden % 8) return MLA_ERR_INVALID_ARG;
+    if (batch == 0 || n_new == 0) return MLA_OK;
+    if (!h || !w_dkv || !w_kr || !start_pos) return MLA_ERR_INVALID_ARG;
+    if (!aligned16(h) || !aligned16(w_dkv) || !aligned16(w_kr)) return MLA_ERR_INVALID_ARG;
+    if (w_q && (!q_nope || !q_pe || !aligned16(w_q) || !aligned16(q_nope) || !aligned16(q_pe)))
+        return MLA_ERR_INVALID_ARG;
+    if (static_cast<int64_t>(batch) * n_new > (1 << 24)) return MLA_ERR_UNSUPPORTED;
+    unsigned *status = nullptr;
+    if ((s = device_info(&status, nullptr)) != MLA_OK) return s;
+    return from_cuda(launch_project(*dims, v, batch, n_new, h, w_dkv, w_kr, w_q, start_pos, q_nope, q_pe, status,
+                                    static_cast<cudaStream_t>(stream)));
+}
+
 mla_status mla_absorb_q(const mla_dims *dims, int32_t batch, int32_t q_len, const void *q_nope, const void *q_pe,
                         const int32_t *kv_len, const void *w_uk, void *q_abs, void *stream)
 {

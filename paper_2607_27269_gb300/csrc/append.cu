@@ -7,10 +7,10 @@ namespace gbmla {
 namespace {
 
 // One block per appended entry (k, b).  The latent row is a bit-exact 16-byte
-// vector copy; the positional key is rotated in fp32 (angle reduced in fp64)
-// and rounded to bf16, nearest-even.
+// vector copy; the positional key is rotated in fp32 (angle reduced exactly
+// as a fixed-point fraction of a turn) and rounded to bf16, nearest-even.
 __global__ void __launch_bounds__(128) cache_append_kernel(CacheView c, int rank, int d_rope, int style,
-                                                          float base, int n_new,
+                                                          const RopeTurns turns, int n_new,
                                                           const uint16_t *__restrict__ c_new,
                                                           const uint16_t *__restrict__ kr_new,
                                                           const int32_t *__restrict__ start_pos,
@@ -47,7 +47,7 @@ __global__ void __launch_bounds__(128) cache_append_kernel(CacheView c, int rank
     const int half = d_rope / 2;
     for (int e = threadIdx.x; e < half; e += blockDim.x) {
         float cs, sn;
-        rope_cos_sin(pos, rope_theta(e, d_rope, base), &cs, &sn);
+        rope_cos_sin(pos, turns.f[e], &cs, &sn);
         const int i0 = style == 0 ? e : 2 * e;
         const int i1 = style == 0 ? e + half : 2 * e + 1;
         const float x0 = bf16_bits_to_float(kr[i0]), x1 = bf16_bits_to_float(kr[i1]);
@@ -65,7 +65,7 @@ cudaError_t launch_append(const mla_dims &d, const CacheView &c, int batch, int 
 {
     dim3 grid(n_new, batch);
     return launch_dependent(cache_append_kernel, grid, dim3(128), 0, st, 1, c, d.rank, d.d_rope, d.rope_style,
-                            d.rope_base, n_new, static_cast<const uint16_t *>(c_new),
+                            rope_turns(d.d_rope, d.rope_base), n_new, static_cast<const uint16_t *>(c_new),
                             static_cast<const uint16_t *>(kr_new), start_pos, status);
 }
 

@@ -8,16 +8,22 @@
 namespace gbmla {
 namespace {
 
-// Block (row group, sequence b).  A row of o_lat is rank floats; `tpr`
-// threads share it, each owning VEC consecutive float4 (so tpr = rank / 4 /
-// VEC), and a 256-thread block covers 256 / tpr rows.  Every partial of the
-// row is read once, with all of them in flight at the same time.
-template <int VEC>
-__global__ void __launch_bounds__(256) combine_kernel(int batch, int q_len, int H, int rank, int max_kv, int S,
-                                                     const int32_t *__restrict__ kv_len,
-                                                     const float *__restrict__ o_part,
-                                                     const float *__restrict__ lse_part, float *o_lat,
-                                                     float *lse_out)
+// Block (row group, sequence b), 128 threads.  A row of o_lat is rank floats;
+// each thread owns one float4 of it (rank / 4 threads per row) in RPT rows
+// (RPT > 1 only when there are rows enough to fill the GPU anyway: it spreads
+// the per-block prologue over more work).  The partials are merged online:
+// KF partitions per step, their log-sum-exps and partial rows all loaded
+// together, the running exponent base raised when a step brings a larger one.
+// An empty partition (fewer tiles than partitions) was never written: its
+// values are loaded (the slot exists) but never used.
+constexpr int kCombineThreads = 128;
+
+template <int RPT, int KF>
+__global__ void __launch_bounds__(kCombineThreads) combine_kernel(int batch, int q_len, int H, int rank, int max_kv,
+                                                                 int S, const int32_t *__restrict__ kv_len,
+                                                                 const float *__restrict__ o_part,
+                                                                 const float *__restrict__ lse_part, float *o_lat,
+                                                                 float *lse_out)
 {
     griddep_wait();
     griddep_launch_dependents();
@@ -29,65 +35,75 @@ __global__ void __launch_bounds__(256) combine_kernel(int batch, int q_len, int 
     if (nb == 0 || T == 0) return;  // invalid length: recorded by the attention kernel
     const int k_first = part_of_tile(t0, T, S), k_last = part_of_tile(t0 + nb - 1, T, S);
     const int rows = q_len * H;
-    const int tpr = rank / (4 * VEC);
-    const int rpb = blockDim.x / tpr;
-    const int row = blockIdx.x * rpb + threadIdx.x / tpr;
+    const int tpr = rank / 4, rpb = kCombineThreads / tpr;
     const int part = threadIdx.x % tpr;
-    if (row >= rows) return;
-    // a partition is empty only when there are fewer tiles than partitions
-    const bool may_be_empty = T < S;
-    auto empty = [&](int k) { return may_be_empty && part_begin(k, T, S) == part_begin(k + 1, T, S); };
-    // exponent base: the largest partial log-sum-exp of the row
-    float m = -INFINITY;
-    for (int k = k_first; k <= k_last; ++k) {
-        if (empty(k)) continue;
-        m = fmaxf(m, lse_part[(static_cast<int64_t>(b) + k) * rows + row]);
+    if (threadIdx.x >= rpb * tpr) return;  // rank / 4 need not divide the block
+    const int row0 = blockIdx.x * rpb * RPT + threadIdx.x / tpr;
+    const bool may_be_empty = T < S;  // a partition is empty only when there are fewer tiles than partitions
+    float m[RPT], wsum[RPT];
+    float4 acc[RPT];
+#pragma unroll
+    for (int r = 0; r < RPT; ++r) {
+        m[r] = -INFINITY;
+        wsum[r] = 0.f;
+        acc[r] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
-    float4 acc[VEC];
+    for (int k0 = k_first; k0 <= k_last; k0 += KF) {
+        float l[RPT][KF];
+        float4 x[RPT][KF];
 #pragma unroll
-    for (int u = 0; u < VEC; ++u) acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-    float wsum = 0.f;
-    if (m != -INFINITY) {
-        // four partitions per step, their loads issued together
-        for (int k4 = k_first; k4 <= k_last; k4 += 4) {
-            float wk[4];
-            float4 x[4][VEC];
+        for (int j = 0; j < KF; ++j) {
+            const int k = k0 + j;
+            const bool live = k <= k_last && !(may_be_empty && part_begin(k, T, S) == part_begin(k + 1, T, S));
+            const int64_t slot = static_cast<int64_t>(b) + (k <= k_last ? k : k_last);
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const int k = k4 + j;
-                wk[j] = 0.f;
-                if (k <= k_last && !empty(k)) {
-                    const int64_t slot = static_cast<int64_t>(b) + k;
-                    const float l = lse_part[slot * rows + row];
-                    if (l != -INFINITY) {
-                        wk[j] = __expf(l - m);
-                        const float4 *src =
-                            reinterpret_cast<const float4 *>(o_part + (slot * rows + row) * rank) + part * VEC;
-#pragma unroll
-                        for (int u = 0; u < VEC; ++u) x[j][u] = __ldcs(src + u);  // read once: do not keep in L2
-                    }
-                }
-            }
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                if (wk[j] == 0.f) continue;
-                wsum += wk[j];
-#pragma unroll
-                for (int u = 0; u < VEC; ++u) {
-                    acc[u].x += wk[j] * x[j][u].x;
-                    acc[u].y += wk[j] * x[j][u].y;
-                    acc[u].z += wk[j] * x[j][u].z;
-                    acc[u].w += wk[j] * x[j][u].w;
+            for (int r = 0; r < RPT; ++r) {
+                const int row = row0 + r * rpb;
+                l[r][j] = -INFINITY;
+                x[r][j] = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (row < rows) {
+                    const float lv = lse_part[slot * rows + row];
+                    x[r][j] = __ldcs(reinterpret_cast<const float4 *>(o_part + (slot * rows + row) * rank) + part);
+                    l[r][j] = live ? lv : -INFINITY;
                 }
             }
         }
-    }
-    const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
-    float4 *dst = reinterpret_cast<float4 *>(o_lat + (static_cast<int64_t>(b) * rows + row) * rank) + part * VEC;
 #pragma unroll
-    for (int u = 0; u < VEC; ++u) dst[u] = make_float4(acc[u].x * inv, acc[u].y * inv, acc[u].z * inv, acc[u].w * inv);
-    if (lse_out && part == 0)
-        lse_out[static_cast<int64_t>(b) * rows + row] = wsum > 0.f ? m + logf(wsum) : -INFINITY;
+        for (int r = 0; r < RPT; ++r) {
+            float bm = l[r][0];
+#pragma unroll
+            for (int j = 1; j < KF; ++j) bm = fmaxf(bm, l[r][j]);
+            if (bm == -INFINITY) continue;
+            const float mn = fmaxf(m[r], bm);
+            const float sc = m[r] == -INFINITY ? 0.f : __expf(m[r] - mn);
+            m[r] = mn;
+            wsum[r] *= sc;
+            acc[r].x *= sc;
+            acc[r].y *= sc;
+            acc[r].z *= sc;
+            acc[r].w *= sc;
+#pragma unroll
+            for (int j = 0; j < KF; ++j) {
+                if (l[r][j] == -INFINITY) continue;  // no key there, or never written
+                const float wk = __expf(l[r][j] - mn);
+                wsum[r] += wk;
+                acc[r].x += wk * x[r][j].x;
+                acc[r].y += wk * x[r][j].y;
+                acc[r].z += wk * x[r][j].z;
+                acc[r].w += wk * x[r][j].w;
+            }
+        }
+    }
+#pragma unroll
+    for (int r = 0; r < RPT; ++r) {
+        const int row = row0 + r * rpb;
+        if (row >= rows) continue;
+        const float inv = wsum[r] > 0.f ? 1.f / wsum[r] : 0.f;
+        reinterpret_cast<float4 *>(o_lat + (static_cast<int64_t>(b) * rows + row) * rank)[part] =
+            make_float4(acc[r].x * inv, acc[r].y * inv, acc[r].z * inv, acc[r].w * inv);
+        if (lse_out && part == 0)
+            lse_out[static_cast<int64_t>(b) * rows + row] = wsum[r] > 0.f ? m[r] + logf(wsum[r]) : -INFINITY;
+    }
 }
 
 }  // namespace
@@ -96,13 +112,20 @@ cudaError_t launch_combine(int batch, int q_len, int num_heads, int rank, int ma
                            const int32_t *kv_len, const float *o_part, const float *lse_part, float *o_lat,
                            float *lse, cudaStream_t st)
 {
-    // rank is a multiple of 64 (<= 512): 2 float4 per thread gives tpr = rank / 8 <= 64
-    const int tpr = rank / 8, rpb = 256 / tpr;
+    // rank is a multiple of 64 (<= 512): rank / 4 <= 128 threads per row
+    const int tpr = rank / 4, rpb = kCombineThreads / tpr;
     const int rows = q_len * num_heads;
-    dim3 grid((rows + rpb - 1) / rpb, batch);
     if (batch == 0 || rows == 0) return cudaSuccess;
-    return launch_dependent(combine_kernel<2>, grid, dim3(256), 0, st, 1, batch, q_len, num_heads, rank, max_kv,
-                            num_splits, kv_len, o_part, lse_part, o_lat, lse);
+    // four rows per thread once that still leaves several blocks per SM
+    const int64_t blocks1 = static_cast<int64_t>((rows + rpb - 1) / rpb) * batch;
+    if (blocks1 >= 16 * 152) {
+        dim3 grid((rows + 4 * rpb - 1) / (4 * rpb), batch);
+        return launch_dependent(combine_kernel<4, 2>, grid, dim3(kCombineThreads), 0, st, 1, batch, q_len, num_heads,
+                                rank, max_kv, num_splits, kv_len, o_part, lse_part, o_lat, lse);
+    }
+    dim3 grid((rows + rpb - 1) / rpb, batch);
+    return launch_dependent(combine_kernel<1, 8>, grid, dim3(kCombineThreads), 0, st, 1, batch, q_len, num_heads, rank,
+                            max_kv, num_splits, kv_len, o_part, lse_part, o_lat, lse);
 }
 
 }  // namespace gbmla

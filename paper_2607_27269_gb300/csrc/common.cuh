@@ -1,6 +1,8 @@
 // Device-side helpers shared by the kernels of libgbmla.so.
 #pragma once
 
+#include <math.h>
+
 #include <utility>
 
 #include <cuda_bf16.h>
@@ -189,20 +191,32 @@ __device__ __forceinline__ void block_tile_sums(const int32_t *kv_len, int n, in
 }
 
 
-// RoPE angle pos * theta_k reduced to [-pi, pi] in fp64 before the fp32
-// sincos, so that positions up to 2^31 keep fp32 accuracy.
-__device__ __forceinline__ void rope_cos_sin(int64_t pos, double theta, float *c, float *s)
+// RoPE frequencies (Sec. 3.1, theta_k = base^(-2k/d_rope)) as fixed-point
+// fractions of a turn, f_k = round(theta_k / (2 pi) * 2^64), computed once on
+// the host.  The angle of position pos is then pos * f_k mod 2^64 turns: one
+// exact integer multiply does the range reduction for any position, and the
+// result, read as a signed fraction x in [-1, 1), is the angle pi * x that
+// sincospif evaluates in fp32.  No fp64 arithmetic runs on the device.
+struct RopeTurns {
+    uint64_t f[32];  // d_rope / 2 <= 32 frequencies
+};
+
+inline RopeTurns rope_turns(int d_rope, float base)
 {
+    RopeTurns t{};
     const double two_pi = 6.283185307179586476925286766559;
-    double ang = static_cast<double>(pos) * theta;
-    ang -= two_pi * rint(ang / two_pi);
-    sincosf(static_cast<float>(ang), s, c);
+    for (int k = 0; k < d_rope / 2 && k < 32; ++k) {
+        const double theta = pow(static_cast<double>(base), -2.0 * k / d_rope);  // <= 1
+        t.f[k] = static_cast<uint64_t>(ldexp(theta / two_pi, 64));                // < 2^62
+    }
+    return t;
 }
 
-// theta_k = base^(-2k/d) in fp64.
-__device__ __forceinline__ double rope_theta(int k, int d, float base)
+__device__ __forceinline__ void rope_cos_sin(int64_t pos, uint64_t f, float *c, float *s)
 {
-    return exp2(-(2.0 * k / d) * log2(static_cast<double>(base)));
+    const uint64_t turn = static_cast<uint64_t>(pos) * f;                                   // mod 2^64
+    const float x = static_cast<float>(static_cast<int64_t>(turn)) * 1.0842021724855044e-19f;  // 2^-63
+    sincospif(x, s, c);
 }
 
 }  // namespace gbmla

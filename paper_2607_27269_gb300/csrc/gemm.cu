@@ -8,6 +8,14 @@
 //
 // All as one tcgen05 GEMM: up to 128 rows x BN columns per CTA, A and the
 // weight tile loaded by TMA, the fp32 accumulator in TMEM.
+//
+// The same kernel, with PROJ set, projects the step's hidden states (the step
+// before the cache append, Sec. 3.2 and Eq. 1): rows are the entries
+// h[b, k, :], and the column tiles run over W^DKV (the latent), one tile for
+// W^KR (the positional key) and W^Q (the queries).  Its epilogue writes the
+// latent row and the positional key, rotated to the entry's position in fp32,
+// straight into the (paged) cache, and splits each query head into its
+// non-positional and positional parts.
 #include <cudaTypedefs.h>
 
 #include "common.cuh"
@@ -20,6 +28,150 @@ namespace {
 __device__ __forceinline__ int64_t phys_row(const GroupGemm &p, int g, int m)
 {
     return static_cast<int64_t>(m / p.hpg) * p.blk + g * p.hpg + m % p.hpg;
+}
+
+// Epilogue arguments of the projection (PROJ): column tiles [0, tiles_lat)
+// hold the latent, tile tiles_lat the positional key, the rest the queries.
+struct ProjEpi {
+    CacheView cache;
+    const int32_t *start_pos;
+    uint16_t *q_nope, *q_pe;
+    int n_new, rank, d_rope, d_nope, heads, style;
+    RopeTurns turns;
+    int tiles_lat;
+    uint32_t box_bytes[3];  // weight-tile bytes of the three column regions
+};
+
+__device__ __forceinline__ void store16_bf16(uint16_t *dst, const uint32_t (&v)[16])
+{
+    uint32_t w[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        const __nv_bfloat162 b = __floats2bfloat162_rn(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1]));
+        w[e] = *reinterpret_cast<const uint32_t *>(&b);
+    }
+    reinterpret_cast<uint4 *>(dst)[0] = make_uint4(w[0], w[1], w[2], w[3]);
+    reinterpret_cast<uint4 *>(dst)[1] = make_uint4(w[4], w[5], w[6], w[7]);
+}
+
+// R_pos of the DR projected positional-key values x (fp32; the angle reduced
+// exactly as a fraction of a turn), rounded once to bf16 into `row`.
+template <int DR>
+__device__ __forceinline__ void rotate_store(const float (&x)[64], int64_t pos, int style, const RopeTurns &turns,
+                                             uint16_t *row)
+{
+    constexpr int HALF = DR / 2;
+    __align__(16) uint16_t y[DR];
+    if (style == 0) {
+#pragma unroll
+        for (int k = 0; k < HALF; ++k) {
+            float cs, sn;
+            rope_cos_sin(pos, turns.f[k], &cs, &sn);
+            y[k] = __bfloat16_as_ushort(__float2bfloat16_rn(x[k] * cs - x[k + HALF] * sn));
+            y[k + HALF] = __bfloat16_as_ushort(__float2bfloat16_rn(x[k + HALF] * cs + x[k] * sn));
+        }
+    } else {
+#pragma unroll
+        for (int k = 0; k < HALF; ++k) {
+            float cs, sn;
+            rope_cos_sin(pos, turns.f[k], &cs, &sn);
+            y[2 * k] = __bfloat16_as_ushort(__float2bfloat16_rn(x[2 * k] * cs - x[2 * k + 1] * sn));
+            y[2 * k + 1] = __bfloat16_as_ushort(__float2bfloat16_rn(x[2 * k + 1] * cs + x[2 * k] * sn));
+        }
+    }
+#pragma unroll
+    for (int v = 0; v < DR / 8; ++v) reinterpret_cast<uint4 *>(row)[v] = reinterpret_cast<const uint4 *>(y)[v];
+}
+
+// Projection epilogue for tile row m (the entry h[m / n_new, m % n_new]);
+// every lane of the warp calls it (the TMEM loads are warp-collective).
+template <int BN>
+__device__ void proj_epilogue(const GroupGemm &p, const ProjEpi &e, uint32_t t_lane, int m, bool row_ok)
+{
+    const int ty = blockIdx.y;
+    if (ty > e.tiles_lat) {
+        // ---- queries: column c of W^Q is element c % dq of head c / dq
+        const int dq = e.d_nope + e.d_rope, nq = e.heads * dq;
+        const int c0 = (ty - e.tiles_lat - 1) * BN;
+#pragma unroll 1
+        for (int j = 0; j < BN; j += 16) {
+            uint32_t v[16];
+            tc::ld_32x32b_x16(t_lane + j, v);
+            tc::wait_ld();
+            const int c = c0 + j;
+            if (!row_ok || c >= nq) continue;
+            const int head = c / dq, el = c % dq;
+            const int64_t hrow = static_cast<int64_t>(m) * e.heads + head;
+            if (c + 16 <= nq && el + 16 <= e.d_nope) {
+                store16_bf16(e.q_nope + hrow * e.d_nope + el, v);
+            } else if (c + 16 <= nq && el >= e.d_nope && el + 16 <= dq) {
+                store16_bf16(e.q_pe + hrow * e.d_rope + (el - e.d_nope), v);
+            } else {
+                for (int u = 0; u < 16 && c + u < nq; ++u) {
+                    const int hu = (c + u) / dq, eu = (c + u) % dq;
+                    const int64_t r = static_cast<int64_t>(m) * e.heads + hu;
+                    const uint16_t b = __bfloat16_as_ushort(__float2bfloat16_rn(__uint_as_float(v[u])));
+                    if (eu < e.d_nope)
+                        e.q_nope[r * e.d_nope + eu] = b;
+                    else
+                        e.q_pe[r * e.d_rope + (eu - e.d_nope)] = b;
+                }
+            }
+        }
+        return;
+    }
+    // ---- the entry's cache row: position start_pos[b] + k, through the block table when paged
+    const CacheView &c = e.cache;
+    bool ok = row_ok;
+    int64_t pos = 0, blk = 0, slot = 0;
+    if (ok) {
+        const int b = m / e.n_new, k = m % e.n_new;
+        pos = static_cast<int64_t>(e.start_pos[b]) + k;
+        ok = pos >= 0 && pos < c.capacity;
+        if (ok && c.block_table) {
+            const int32_t page = c.block_table[static_cast<int64_t>(b) * c.bt_stride + pos / c.page_size];
+            ok = page >= 0 && page < c.num_pages;
+            blk = page;
+            slot = pos % c.page_size;
+        } else {
+            blk = b;
+            slot = pos;
+        }
+        if (!ok) record_status(p.status, kStatusBounds);
+    }
+    if (ty < e.tiles_lat) {
+        // ---- latent c = W^DKV h, rounded once
+        uint16_t *crow = static_cast<uint16_t *>(const_cast<void *>(c.c_kv)) + blk * c.c_blk + slot * c.c_tok;
+#pragma unroll 1
+        for (int j = 0; j < BN; j += 16) {
+            uint32_t v[16];
+            tc::ld_32x32b_x16(t_lane + j, v);
+            tc::wait_ld();
+            if (ok) store16_bf16(crow + ty * BN + j, v);
+        }
+        return;
+    }
+    // ---- positional key R_pos W^KR h (d_rope = 32 or 64 columns of this tile)
+    float x[64];
+#pragma unroll
+    for (int j = 0; j < 64; j += 16) {
+        if (j < e.d_rope) {
+            uint32_t v[16];
+            tc::ld_32x32b_x16(t_lane + j, v);
+            tc::wait_ld();
+#pragma unroll
+            for (int u = 0; u < 16; ++u) x[j + u] = __uint_as_float(v[u]);
+        } else {
+#pragma unroll
+            for (int u = 0; u < 16; ++u) x[j + u] = 0.f;
+        }
+    }
+    if (!ok) return;
+    uint16_t *rrow = static_cast<uint16_t *>(const_cast<void *>(c.k_rope)) + blk * c.r_blk + slot * c.r_tok;
+    if (e.d_rope == 64)
+        rotate_store<64>(x, pos, e.style, e.turns, rrow);
+    else
+        rotate_store<32>(x, pos, e.style, e.turns, rrow);
 }
 
 // ---------------------------------------------------------------- tensor-core GEMM
@@ -46,11 +198,16 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap *map
 }
 
 // BN: columns per CTA.  NMAJ: the weight is N-major.  AF32: A is fp32.
-template <int BN, bool NMAJ, bool AF32>
+// PROJ: the projection (K-major weights map_b, map_b2, map_b3 by column region).
+template <int BN, bool NMAJ, bool AF32, bool PROJ>
 __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_constant__ GroupGemm p,
                                                                const __grid_constant__ CUtensorMap map_a,
-                                                               const __grid_constant__ CUtensorMap map_b)
+                                                               const __grid_constant__ CUtensorMap map_b,
+                                                               const __grid_constant__ CUtensorMap map_b2,
+                                                               const __grid_constant__ CUtensorMap map_b3,
+                                                               const __grid_constant__ ProjEpi pe)
 {
+    static_assert(!PROJ || (!NMAJ && !AF32), "the projection reads bf16 h and K-major weights");
     constexpr int kABytes = 128 * 128;     // 128 rows x 64 K, bf16, SW128 K-major
     constexpr int kRawBytes = AF32 ? 2 * 128 * 128 : 0;  // two 32-column fp32 boxes
     constexpr int kBBytes = BN * 128;      // BN x 64 K (K-major) or 64 K x BN (N-major)
@@ -100,9 +257,18 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
 
     if (warp == 0) {
         // ---- A and weight tiles by TMA
+        const CUtensorMap *mb = &map_b;
+        int brow = g * p.N + n0;
+        uint32_t bbytes = kBBytes;
+        if (PROJ) {
+            const int ty = blockIdx.y, region = ty < pe.tiles_lat ? 0 : ty == pe.tiles_lat ? 1 : 2;
+            mb = region == 0 ? &map_b : region == 1 ? &map_b2 : &map_b3;
+            brow = region == 0 ? n0 : region == 1 ? 0 : (ty - pe.tiles_lat - 1) * BN;
+            bbytes = pe.box_bytes[region];
+        }
         if (lane == 0) {
             tc::prefetch_tensormap(&map_a);
-            tc::prefetch_tensormap(&map_b);
+            tc::prefetch_tensormap(mb);
         }
         for (int c = 0; c < nk; ++c) {
             const int s = c % NS, round = c / NS;
@@ -112,14 +278,14 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
             }
             if (lane == 0) {
                 const uint32_t fb = smem_u32(&bars.full[s]);
-                tc::mbar_arrive_expect_tx(fb, kBBytes + (AF32 ? 0u : a_bytes));
+                tc::mbar_arrive_expect_tx(fb, bbytes + (AF32 ? 0u : a_bytes));
                 const uint32_t dst = smem_u32(sb + s * kBBytes);
                 if (NMAJ) {
                     // rows = K of group g, columns = N: one 64 x 64 box per 64 columns
                     for (int j = 0; j < BN / 64; ++j)
                         tc::tma_load_2d(dst + j * 64 * 128, &map_b, n0 + 64 * j, g * p.K + 64 * c, fb);
                 } else {
-                    tc::tma_load_2d(dst, &map_b, 64 * c, g * p.N + n0, fb);
+                    tc::tma_load_2d(dst, mb, 64 * c, brow, fb);
                 }
                 if (AF32) {
                     const uint32_t rb = smem_u32(&bars.raw_full[s]);
@@ -203,6 +369,9 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
             const bool row_ok = i < RT && me < p.M;
             const uint32_t t_lane = tmem + (static_cast<uint32_t>(q * 32) << 16);
             const int64_t orow = row_ok ? phys_row(p, g, me) : 0;
+            if (PROJ) {
+                proj_epilogue<BN>(p, pe, t_lane, me, row_ok);
+            } else {
 #pragma unroll 1
             for (int j = 0; j < BN; j += 16) {
                 uint32_t v[16];
@@ -212,18 +381,12 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
                 if (!row_ok || n >= p.N) continue;
                 uint16_t *dst = static_cast<uint16_t *>(p.C) + orow * p.ldc + n;
                 if (n + 16 <= p.N) {
-                    uint32_t w[8];
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const __nv_bfloat162 b = __floats2bfloat162_rn(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1]));
-                        w[e] = *reinterpret_cast<const uint32_t *>(&b);
-                    }
-                    reinterpret_cast<uint4 *>(dst)[0] = make_uint4(w[0], w[1], w[2], w[3]);
-                    reinterpret_cast<uint4 *>(dst)[1] = make_uint4(w[4], w[5], w[6], w[7]);
+                    store16_bf16(dst, v);
                 } else {
                     for (int e = 0; e < 16 && n + e < p.N; ++e)
                         dst[e] = __bfloat16_as_ushort(__float2bfloat16_rn(__uint_as_float(v[e])));
                 }
+            }
             }
         }
     }
@@ -237,72 +400,154 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode_gemm = nullptr;
 
-template <int BN, bool NMAJ, bool AF32>
-cudaError_t launch_tc(const GroupGemm &p, cudaStream_t st)
+cudaError_t get_encoder()
 {
-    if (!g_encode_gemm) {
-        cudaDriverEntryPointQueryResult q;
-        void *fn = nullptr;
-        cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
-        if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn) return e != cudaSuccess ? e : cudaErrorNotSupported;
-        g_encode_gemm = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
-    }
-    if (p.hpg < 1 || p.hpg > 128 || p.M % p.hpg) return cudaErrorInvalidValue;
-    const int es = AF32 ? 4 : 2;
-    // row blocks per tile: as many as fit 128 rows, but no more than there are
-    // (a short A box leaves the tile's other rows stale; their results are dropped)
-    const int rblk = (128 / p.hpg) < (p.M / p.hpg) ? (128 / p.hpg) : (p.M / p.hpg);
-    CUtensorMap ma, mb;
-    {   // A: (K, head in group, group, row block) with the row mapping's strides
-        cuuint64_t dims[4] = {static_cast<cuuint64_t>(p.K), static_cast<cuuint64_t>(p.hpg),
-                              static_cast<cuuint64_t>(p.G), static_cast<cuuint64_t>(p.M / p.hpg)};
-        cuuint64_t strides[3] = {static_cast<cuuint64_t>(p.lda) * es, static_cast<cuuint64_t>(p.hpg) * p.lda * es,
-                                 static_cast<cuuint64_t>(p.blk) * p.lda * es};
-        cuuint32_t box[4] = {AF32 ? 32u : 64u, static_cast<cuuint32_t>(p.hpg), 1u, static_cast<cuuint32_t>(rblk)};
-        cuuint32_t es4[4] = {1, 1, 1, 1};
-        CUresult r = g_encode_gemm(&ma, AF32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4,
-                                   const_cast<void *>(p.A), dims, strides, box, es4, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                                   CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-        if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
-    }
-    {
-        cuuint64_t dims[2], strides[1];
-        cuuint32_t box[2], es2[2] = {1, 1};
-        if (NMAJ) {  // [G K rows][N columns]
-            dims[0] = static_cast<cuuint64_t>(p.N);
-            dims[1] = static_cast<cuuint64_t>(p.G) * p.K;
-            strides[0] = static_cast<cuuint64_t>(p.N) * 2;
-            box[0] = 64;
-            box[1] = 64;
-        } else {     // [G N rows][K columns]
-            dims[0] = static_cast<cuuint64_t>(p.K);
-            dims[1] = static_cast<cuuint64_t>(p.G) * p.N;
-            strides[0] = static_cast<cuuint64_t>(p.K) * 2;
-            box[0] = 64;
-            box[1] = BN;
-        }
-        CUresult r = g_encode_gemm(&mb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(p.B), dims, strides,
-                                   box, es2, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-        if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
-    }
-    const int nk = (p.K + 63) / 64;
+    if (g_encode_gemm) return cudaSuccess;
+    cudaDriverEntryPointQueryResult q;
+    void *fn = nullptr;
+    cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn) return e != cudaSuccess ? e : cudaErrorNotSupported;
+    g_encode_gemm = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    return cudaSuccess;
+}
+
+// A: (K, head in group, group, row block) with the row mapping's strides.
+bool encode_a(const GroupGemm &p, int rblk, bool f32, CUtensorMap *ma)
+{
+    const int es = f32 ? 4 : 2;
+    cuuint64_t dims[4] = {static_cast<cuuint64_t>(p.K), static_cast<cuuint64_t>(p.hpg), static_cast<cuuint64_t>(p.G),
+                          static_cast<cuuint64_t>(p.M / p.hpg)};
+    cuuint64_t strides[3] = {static_cast<cuuint64_t>(p.lda) * es, static_cast<cuuint64_t>(p.hpg) * p.lda * es,
+                             static_cast<cuuint64_t>(p.blk) * p.lda * es};
+    cuuint32_t box[4] = {f32 ? 32u : 64u, static_cast<cuuint32_t>(p.hpg), 1u, static_cast<cuuint32_t>(rblk)};
+    cuuint32_t es4[4] = {1, 1, 1, 1};
+    return g_encode_gemm(ma, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4,
+                         const_cast<void *>(p.A), dims, strides, box, es4, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                         CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// A K-major weight [rows][K] in boxes of 64 K x box_rows rows.
+bool encode_kmajor(const void *w, int64_t rows, int K, int box_rows, CUtensorMap *mb)
+{
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(rows)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
+    cuuint32_t box[2] = {64u, static_cast<cuuint32_t>(box_rows)}, es2[2] = {1, 1};
+    return g_encode_gemm(mb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(w), dims, strides, box, es2,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Row blocks per tile: as many as fit 128 rows, but no more than there are
+// (a short A box leaves the tile's other rows stale; their results are dropped).
+int rows_per_tile(const GroupGemm &p) { return (128 / p.hpg) < (p.M / p.hpg) ? (128 / p.hpg) : (p.M / p.hpg); }
+
+// Ring depth: as many stages as fit 192 KB, at most kStages and the K chunks.
+template <int BN, bool AF32>
+int ring_stages(int K, size_t *smem)
+{
+    const int nk = (K + 63) / 64;
     const size_t per_stage = 128 * 128 + BN * 128 + (AF32 ? 2 * 128 * 128 : 0);
     int ns = static_cast<int>((192 * 1024) / per_stage);
     if (ns > kStages) ns = kStages;
     if (ns > nk) ns = nk;
     if (ns < 1) ns = 1;
+    *smem = 1024 + static_cast<size_t>(ns) * per_stage;
+    return ns;
+}
+
+template <int BN, bool NMAJ, bool AF32>
+cudaError_t launch_tc(const GroupGemm &p, cudaStream_t st)
+{
+    cudaError_t e = get_encoder();
+    if (e != cudaSuccess) return e;
+    if (p.hpg < 1 || p.hpg > 128 || p.M % p.hpg) return cudaErrorInvalidValue;
+    const int rblk = rows_per_tile(p);
+    CUtensorMap ma, mb;
+    if (!encode_a(p, rblk, AF32, &ma)) return cudaErrorInvalidValue;
+    if (NMAJ) {  // [G K rows][N columns], 64 x 64 boxes
+        cuuint64_t dims[2] = {static_cast<cuuint64_t>(p.N), static_cast<cuuint64_t>(p.G) * p.K};
+        cuuint64_t strides[1] = {static_cast<cuuint64_t>(p.N) * 2};
+        cuuint32_t box[2] = {64u, 64u}, es2[2] = {1, 1};
+        CUresult r = g_encode_gemm(&mb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(p.B), dims, strides,
+                                   box, es2, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    } else if (!encode_kmajor(p.B, static_cast<int64_t>(p.G) * p.N, p.K, BN, &mb)) {  // [G N rows][K columns]
+        return cudaErrorInvalidValue;
+    }
+    size_t smem = 0;
     GroupGemm q = p;
-    q.stages = ns;
+    q.stages = ring_stages<BN, AF32>(p.K, &smem);
     q.rblk = rblk;
-    const size_t smem = 1024 + static_cast<size_t>(ns) * per_stage;
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, NMAJ, AF32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
+    e = cudaFuncSetAttribute(gemm_tc_kernel<BN, NMAJ, AF32, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     const int rt = rblk * p.hpg;
     dim3 grid((p.M + rt - 1) / rt, (p.N + BN - 1) / BN, p.G);
-    return launch_dependent(gemm_tc_kernel<BN, NMAJ, AF32>, grid, dim3(kGemmThreads), smem, st, 1, q, ma, mb);
+    ProjEpi none{};
+    return launch_dependent(gemm_tc_kernel<BN, NMAJ, AF32, false>, grid, dim3(kGemmThreads), smem, st, 1, q, ma, mb,
+                            mb, mb, none);
+}
+
+// The projection: h [M = batch n_new, hidden] against W^DKV (rank rows), W^KR
+// (d_rope rows, one column tile) and W^Q (H (d_nope + d_rope) rows, or none).
+template <int BN>
+cudaError_t launch_proj(const mla_dims &d, const CacheView &c, int batch, int n_new, const void *h,
+                        const void *w_dkv, const void *w_kr, const void *w_q, const int32_t *start_pos, void *q_nope,
+                        void *q_pe, unsigned *status, cudaStream_t st)
+{
+    cudaError_t e = get_encoder();
+    if (e != cudaSuccess) return e;
+    GroupGemm p{};
+    p.M = batch * n_new;
+    p.K = d.hidden;
+    p.G = 1;
+    p.hpg = 1;
+    p.blk = 1;
+    p.A = h;
+    p.a_f32 = 0;
+    p.lda = d.hidden;
+    p.status = status;
+    const int nq = w_q ? d.num_heads * (d.d_nope + d.d_rope) : 0;
+    const int rope_rows = d.d_rope < BN ? d.d_rope : BN, q_rows = nq < BN ? nq : BN;
+    ProjEpi pe{};
+    pe.cache = c;
+    pe.start_pos = start_pos;
+    pe.q_nope = static_cast<uint16_t *>(q_nope);
+    pe.q_pe = static_cast<uint16_t *>(q_pe);
+    pe.n_new = n_new;
+    pe.rank = d.rank;
+    pe.d_rope = d.d_rope;
+    pe.d_nope = d.d_nope;
+    pe.heads = d.num_heads;
+    pe.style = d.rope_style;
+    pe.turns = rope_turns(d.d_rope, d.rope_base);
+    pe.tiles_lat = d.rank / BN;
+    pe.box_bytes[0] = BN * 128;
+    pe.box_bytes[1] = static_cast<uint32_t>(rope_rows) * 128;
+    pe.box_bytes[2] = static_cast<uint32_t>(q_rows) * 128;
+    const int rblk = rows_per_tile(p);
+    CUtensorMap ma, m0, m1, m2;
+    if (!encode_a(p, rblk, false, &ma) || !encode_kmajor(w_dkv, d.rank, d.hidden, BN, &m0) ||
+        !encode_kmajor(w_kr, d.d_rope, d.hidden, rope_rows, &m1))
+        return cudaErrorInvalidValue;
+    if (w_q) {
+        if (!encode_kmajor(w_q, nq, d.hidden, q_rows, &m2)) return cudaErrorInvalidValue;
+    } else {
+        m2 = m0;  // never read: no query tiles
+    }
+    const int tiles = pe.tiles_lat + 1 + (nq + BN - 1) / BN;
+    p.N = tiles * BN;
+    size_t smem = 0;
+    p.stages = ring_stages<BN, false>(p.K, &smem);
+    p.rblk = rblk;
+    e = cudaFuncSetAttribute(gemm_tc_kernel<BN, false, false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    dim3 grid((p.M + rblk - 1) / rblk, tiles, 1);
+    return launch_dependent(gemm_tc_kernel<BN, false, false, true>, grid, dim3(kGemmThreads), smem, st, 1, p, ma, m0,
+                            m1, m2, pe);
 }
 
 }  // namespace
@@ -319,6 +564,18 @@ cudaError_t launch_group_gemm(const GroupGemm &p, cudaStream_t st)
     }
     if (p.b_nmajor) return narrow ? launch_tc<64, true, false>(p, st) : launch_tc<128, true, false>(p, st);
     return narrow ? launch_tc<64, false, false>(p, st) : launch_tc<128, false, false>(p, st);
+}
+
+cudaError_t launch_project(const mla_dims &d, const CacheView &c, int batch, int n_new, const void *h,
+                           const void *w_dkv, const void *w_kr, const void *w_q, const int32_t *start_pos,
+                           void *q_nope, void *q_pe, unsigned *status, cudaStream_t st)
+{
+    if (batch <= 0 || n_new <= 0) return cudaSuccess;
+    // 128-column tiles once there are enough rows to be tensor-bound and the
+    // latent splits into whole 128-column tiles; 64 otherwise
+    if (batch * n_new > 32 && d.rank % 128 == 0)
+        return launch_proj<128>(d, c, batch, n_new, h, w_dkv, w_kr, w_q, start_pos, q_nope, q_pe, status, st);
+    return launch_proj<64>(d, c, batch, n_new, h, w_dkv, w_kr, w_q, start_pos, q_nope, q_pe, status, st);
 }
 
 }  // namespace gbmla

@@ -78,6 +78,14 @@ struct GroupGemm {
 };
 cudaError_t launch_group_gemm(const GroupGemm &p, cudaStream_t st);
 
+// Projection of the step's hidden states (mla_project_append): one GEMM of
+// h [batch * n_new, hidden] with the three weights side by side, whose
+// epilogue writes the latent rows and the rotated positional keys into the
+// cache and the two query parts to q_nope / q_pe.
+cudaError_t launch_project(const mla_dims &d, const CacheView &c, int batch, int n_new, const void *h,
+                           const void *w_dkv, const void *w_kr, const void *w_q, const int32_t *start_pos,
+                           void *q_nope, void *q_pe, unsigned *status, cudaStream_t st);
+
 cudaError_t launch_selftest_wait(int64_t limit_ns, unsigned *status, cudaStream_t st);
 
 }  // namespace gbmla

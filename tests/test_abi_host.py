@@ -93,3 +93,26 @@ def test_other_arguments_are_checked_on_the_host():
     # out_proj with W_O needs `out`
     dd = _dims(hidden=256).c()
     assert L.mla_out_proj(ctypes.byref(dd), 1, 1, 16, 16, 16, 16, None, None) == abi.MLA_ERR_INVALID_ARG
+
+
+def test_projection_arguments_are_checked_on_the_host():
+    L = abi.lib()
+    c = abi.MlaCache(0x1000, 0x2000, 512, 64, 512 * 64, 64 * 64, None, 0, 0, 0, 64)
+    # the projection needs the model width
+    d0 = _dims(hidden=0).c()
+    assert L.mla_project_append(ctypes.byref(d0), ctypes.byref(c), 1, 1, 16, 16, 16, None, 16, None, None,
+                                None) == abi.MLA_ERR_INVALID_ARG
+    d = _dims(hidden=256).c()
+    dodd = _dims(hidden=252).c()                                    # row stride not a multiple of 16 bytes
+    assert L.mla_project_append(ctypes.byref(dodd), ctypes.byref(c), 1, 1, 16, 16, 16, None, 16, None, None,
+                                None) == abi.MLA_ERR_INVALID_ARG
+    # missing or misaligned inputs; W_Q without query outputs
+    assert L.mla_project_append(ctypes.byref(d), ctypes.byref(c), 1, 1, None, 16, 16, None, 16, None, None,
+                                None) == abi.MLA_ERR_INVALID_ARG
+    assert L.mla_project_append(ctypes.byref(d), ctypes.byref(c), 1, 1, 24, 16, 16, None, 16, None, None,
+                                None) == abi.MLA_ERR_INVALID_ARG
+    assert L.mla_project_append(ctypes.byref(d), ctypes.byref(c), 1, 1, 16, 16, 16, 16, 16, None, None,
+                                None) == abi.MLA_ERR_INVALID_ARG
+    # an empty batch is a no-op
+    assert L.mla_project_append(ctypes.byref(d), ctypes.byref(c), 0, 1, None, None, None, None, None, None, None,
+                                None) == abi.MLA_OK

@@ -201,3 +201,15 @@ def test_projection_ragged_rows(name, batch):
     assert_close(bf16_to_f64(bits(step.o.cpu())), ref["o"], "o")
     if w.w_o is not None:
         assert_close(bf16_to_f64(bits(step.out.cpu())), ref["out"], "out")
+
+
+def test_rank_that_is_not_a_multiple_of_128():
+    """A latent rank of 192 (a multiple of 64 only) runs the CUDA-core
+    attention kernel and a combine whose rows do not fill its blocks."""
+    s = wl.Shape("rank192", 5, 8, 2, 64, 32, 64, 192, 256, 2, 100, 400)
+    w = wl.make(s, seed=39)
+    step = run_step(abi.to_device(w), num_splits=6)
+    ref = oracle_step(w)
+    assert_close(step.o_lat.cpu().numpy(), ref["o_lat"], "o_lat")
+    assert_close(step.lse.cpu().numpy(), ref["lse"], "lse")
+    assert_close(bf16_to_f64(bits(step.out.cpu())), ref["out"], "out")
