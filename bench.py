@@ -250,19 +250,32 @@ def run_ours(args, rank, world, local):
 
         proj = measure_projection(args, w, dws, stream, dev, l2, peaks=load_peaks())
 
-        # ---- end to end through the public API with host buffers
-        host_in = {k: getattr(w, k).pin_memory() for k in ("q_nope", "q_pe", "c_new", "kr_new", "kv_len", "start_pos")}
+        # ---- end to end through the public API with host buffers: the step's
+        # inputs (queries, new entries, lengths, positions) packed in one pinned
+        # host buffer, copied in one transfer to a device buffer whose views the
+        # step reads; the step's output read back in one transfer
+        names = ("q_nope", "q_pe", "c_new", "kr_new", "kv_len", "start_pos")
+        layout, off = [], 0
+        for k in names:
+            t = getattr(w, k)
+            nbytes = t.numel() * t.element_size()
+            layout.append((k, off, t.dtype, tuple(t.shape), nbytes))
+            off = (off + nbytes + 255) // 256 * 256
+        host_pack = torch.empty(off, dtype=torch.uint8).pin_memory()
+        for k, o, dt, sh, nb in layout:
+            host_pack[o:o + nb].copy_(getattr(w, k).contiguous().view(-1).view(torch.uint8))
+        dev_packs = [torch.empty(off, dtype=torch.uint8, device=dev) for _ in range(replicas)]
+        views = [{k: dp[o:o + nb].view(dt).view(sh) for k, o, dt, sh, nb in layout} for dp in dev_packs]
         out_dev = steps[0].out if steps[0].out is not None else steps[0].o
         host_out = torch.empty(out_dev.shape, dtype=out_dev.dtype).pin_memory()
-        h2d = sum(t.numel() * t.element_size() for t in host_in.values())
+        h2d = off
         d2h = host_out.numel() * host_out.element_size()
 
         def e2e_step(i):
-            d, st = dws[i % replicas], steps[i % replicas]
-            for k, t in host_in.items():
-                getattr(d, k).copy_(t, non_blocking=True)
-            res = st(d.q_nope, d.q_pe, d.kv_len, d.w_uk, d.w_uv, d.w_o, c_new=d.c_new, kr_new=d.kr_new,
-                     start_pos=d.start_pos)
+            d, st, v = dws[i % replicas], steps[i % replicas], views[i % replicas]
+            dev_packs[i % replicas].copy_(host_pack, non_blocking=True)
+            res = st(v["q_nope"], v["q_pe"], v["kv_len"], d.w_uk, d.w_uv, d.w_o, c_new=v["c_new"],
+                     kr_new=v["kr_new"], start_pos=v["start_pos"])
             host_out.copy_(res, non_blocking=True)
 
         for i in range(3):

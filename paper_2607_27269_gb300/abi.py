@@ -254,16 +254,29 @@ class DecodeStep:
 
     def __call__(self, q_nope, q_pe, kv_len, w_uk, w_uv, w_o=None, c_new=None, kr_new=None, start_pos=None,
                  stream=None):
-        d = self.dims
+        # the layer's descriptors and the step's own buffers are fixed: marshal
+        # them once, so that a step costs the five library calls and little else
+        if getattr(self, "_fixed", None) is None:
+            self._structs = (self.dims.c(), self.cache.c())  # kept alive for the references below
+            self._fixed = (ctypes.byref(self._structs[0]), ctypes.byref(self._structs[1]), self.q_abs.data_ptr(),
+                           self.o_part.data_ptr(), self.lse_part.data_ptr(), self.o_lat.data_ptr(),
+                           self.lse.data_ptr(), self.o.data_ptr(),
+                           self.out.data_ptr() if self.out is not None else None)
+        dims, cache, qa, op, lp, ol, ls, o, out = self._fixed
+        d, L, sp = self.dims, lib(), _stream(stream)
+        B, q = self.batch, self.q_len
         if c_new is not None:
-            cache_append(d, self.cache, c_new, kr_new, start_pos, stream)
-        absorb_q(d, q_nope, q_pe, kv_len, w_uk, self.q_abs, stream)
-        decode_attn(d, self.cache, kv_len, self.max_kv_len, self.q_abs, self.o_part, self.lse_part, self.num_splits,
-                    stream)
-        combine(d, self.batch, self.q_len, kv_len, self.max_kv_len, self.o_part, self.lse_part, self.o_lat, self.lse,
-                self.num_splits, stream)
-        out_proj(d, self.o_lat, w_uv, w_o if d.hidden else None, self.o, self.out if d.hidden else None, stream)
-        return self.out if (d.hidden and w_o is not None) else self.o
+            _check("mla_cache_append", L.mla_cache_append(dims, cache, B, c_new.shape[1], _p(c_new), _p(kr_new),
+                                                          _p(start_pos), sp))
+        kv = _p(kv_len)
+        _check("mla_absorb_q", L.mla_absorb_q(dims, B, q, _p(q_nope), _p(q_pe), kv, _p(w_uk), qa, sp))
+        _check("mla_decode_attn", L.mla_decode_attn(dims, cache, B, q, kv, self.max_kv_len, qa, self.num_splits, op,
+                                                    lp, sp))
+        _check("mla_combine", L.mla_combine(dims, B, q, self.num_splits, kv, self.max_kv_len, op, lp, ol, ls, sp))
+        with_o = d.hidden and w_o is not None
+        _check("mla_out_proj", L.mla_out_proj(dims, B, q, ol, _p(w_uv), _p(w_o) if with_o else None, o,
+                                              out if with_o else None, sp))
+        return self.out if with_o else self.o
 
     def from_hidden(self, h, w_dkv, w_kr, w_q, start_pos, kv_len, w_uk, w_uv, w_o=None, stream=None):
         """The step fed by hidden states h [B, q_len, hidden]: the projection

@@ -7,7 +7,11 @@
 // rows of group g, with phys(g, m) = (m / hpg) * blk + g * hpg + m % hpg.
 //
 // All as one tcgen05 GEMM: up to 128 rows x BN columns per CTA, A and the
-// weight tile loaded by TMA, the fp32 accumulator in TMEM.
+// weight tile loaded by TMA, the fp32 accumulator in TMEM.  A GEMM whose tiles
+// would occupy few SMs (few rows, deep K: the output projection of a small
+// batch) splits K over a cluster of up to four CTAs; each leaves its partial
+// tile in shared memory and the cluster sums the partials in a fixed order
+// through distributed shared memory, so the result does not depend on timing.
 //
 // The same kernel, with PROJ set, projects the step's hidden states (the step
 // before the cache append, Sec. 3.2 and Eq. 1): rows are the entries
@@ -218,13 +222,16 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
     unsigned char *smem = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                             ~static_cast<uintptr_t>(1023));
     const int nk = (p.K + 63) / 64;
-    const int NS = p.stages;                             // ring stages (<= kStages, <= nk)
+    const int ks = PROJ ? 1 : p.ksplit;                  // CTAs of the cluster sharing the K range
+    const int kz = blockIdx.x % ks;                      // this CTA's share: chunks [c_begin, c_end)
+    const int c_begin = kz * nk / ks, nkl = (kz + 1) * nk / ks - c_begin;
+    const int NS = p.stages;                             // ring stages (<= kStages)
     unsigned char *sa = smem;                            // NS x A tile
     unsigned char *sb = sa + NS * kABytes;               // NS x B tile
     unsigned char *sr = sb + NS * kBBytes;               // NS x raw fp32 A (AF32)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int R = p.rblk, RT = R * p.hpg;                // row blocks and rows per tile (<= 128)
-    const int mt = blockIdx.x, n0 = blockIdx.y * BN, g = blockIdx.z;
+    const int mt = blockIdx.x / ks, n0 = blockIdx.y * BN, g = blockIdx.z;
     const int m0 = mt * RT;
     const uint32_t a_bytes = static_cast<uint32_t>(RT) * 128;  // per 64-column (bf16) or 32-column (fp32) box
     const uint64_t lim = kWaitLimitNs;
@@ -254,6 +261,7 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
         record_status(p.status, kStatusTimeout);
         fail = 1;
     };
+    bool ep_ok = false;  // split K: this epilogue thread saw its CTA's MMAs complete
 
     if (warp == 0) {
         // ---- A and weight tiles by TMA
@@ -270,8 +278,8 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
             tc::prefetch_tensormap(&map_a);
             tc::prefetch_tensormap(mb);
         }
-        for (int c = 0; c < nk; ++c) {
-            const int s = c % NS, round = c / NS;
+        for (int cc = 0; cc < nkl; ++cc) {
+            const int c = c_begin + cc, s = cc % NS, round = cc / NS;
             if (round >= 1 && !__all_sync(0xffffffffu, mbar_wait(smem_u32(&bars.empty[s]), (round - 1) & 1, lim))) {
                 if (lane == 0) bail();
                 break;
@@ -309,8 +317,8 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
             return tmpl | static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
         };
         bool ok = true;
-        for (int c = 0; c < nk && ok; ++c) {
-            const int s = c % NS, par = (c / NS) & 1;
+        for (int cc = 0; cc < nkl && ok; ++cc) {
+            const int s = cc % NS, par = (cc / NS) & 1;
             ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&bars.full[s]), par, lim) &&
                                              (!AF32 || mbar_wait(smem_u32(&bars.conv_done[s]), par, lim)));
             if (!ok) break;
@@ -320,7 +328,7 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
             for (int kk = 0; kk < 4; ++kk) {
                 const uint32_t b_addr = NMAJ ? b_base + kk * 16 * 128 : b_base + kk * 32;
                 tc::mma_bf16_elect(tmem, with_addr(da, a_base + kk * 32), with_addr(db, b_addr), idesc,
-                                   (c | kk) != 0);
+                                   (cc | kk) != 0);
             }
             tc::commit_elect(smem_u32(&bars.empty[s]));
         }
@@ -330,8 +338,8 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
         if (AF32) {
             // ---- fp32 -> bf16: thread r converts tile row r (two 128-byte swizzled fp32 rows)
             const int r = tid - 64;
-            for (int c = 0; c < nk; ++c) {
-                const int s = c % NS, par = (c / NS) & 1;
+            for (int cc = 0; cc < nkl; ++cc) {
+                const int s = cc % NS, par = (cc / NS) & 1;
                 if (!__all_sync(0xffffffffu, mbar_wait(smem_u32(&bars.raw_full[s]), par, lim))) {
                     if (lane == 0) bail();
                     break;
@@ -371,6 +379,8 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
             const int64_t orow = row_ok ? phys_row(p, g, me) : 0;
             if (PROJ) {
                 proj_epilogue<BN>(p, pe, t_lane, me, row_ok);
+            } else if (ks > 1) {
+                ep_ok = true;  // the partial is pushed once the whole cluster is past its MMAs
             } else {
 #pragma unroll 1
             for (int j = 0; j < BN; j += 16) {
@@ -389,6 +399,63 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
             }
             }
         }
+    }
+    if (!PROJ && ks > 1) {
+        // (1) every CTA of the cluster is past its MMAs, so every ring is free;
+        // (2) push this CTA's partial of each column slice to the slice's owner:
+        // CTA o owns columns [o cw, (o + 1) cw) and receives, in its ring,
+        // recv[r][row][cw + 4] from every rank r; (3) each owner sums its slice
+        // in rank order (four columns per step) and stores the bf16 result
+        const int cw = BN / ks;
+        tc::cluster_sync();
+        if (warp >= 2 && ep_ok && !fail) {
+            tc::fence_after_sync();
+            const int q = warp & 3, i = q * 32 + lane;
+            const uint32_t t_lane = tmem + (static_cast<uint32_t>(q * 32) << 16);
+            const uint32_t recv = smem_u32(smem);
+#pragma unroll 1
+            for (int j = 0; j < BN; j += 16) {
+                uint32_t v[16];
+                tc::ld_32x32b_x16(t_lane + j, v);
+                tc::wait_ld();
+                if (i < RT) {
+                    const int o = j / cw;
+                    const uint32_t local = recv + static_cast<uint32_t>(((kz * RT + i) * (cw + 4) + (j - o * cw)) * 4);
+                    uint32_t remote;
+                    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local), "r"(o));
+#pragma unroll
+                    for (int e = 0; e < 4; ++e)
+                        asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(remote + 16 * e),
+                                     "f"(__uint_as_float(v[4 * e])), "f"(__uint_as_float(v[4 * e + 1])),
+                                     "f"(__uint_as_float(v[4 * e + 2])), "f"(__uint_as_float(v[4 * e + 3]))
+                                     : "memory");
+                }
+            }
+        }
+        tc::cluster_sync();
+        if (warp >= 2 && !fail) {
+            const int q4 = cw / 4;
+            const float *recv = reinterpret_cast<const float *>(smem);
+            for (int idx = tid - 64; idx < RT * q4; idx += 128) {
+                const int i = idx / q4, c4 = (idx % q4) * 4;
+                const int me = m0 + i, n = n0 + kz * cw + c4;
+                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int r = 0; r < ks; ++r) {
+                    const float4 v = *reinterpret_cast<const float4 *>(recv + (r * RT + i) * (cw + 4) + c4);
+                    acc.x += v.x;
+                    acc.y += v.y;
+                    acc.z += v.z;
+                    acc.w += v.w;
+                }
+                if (me >= p.M) continue;
+                uint16_t *dst = static_cast<uint16_t *>(p.C) + phys_row(p, g, me) * p.ldc + n;
+                const float a[4] = {acc.x, acc.y, acc.z, acc.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    if (n + e < p.N) dst[e] = __bfloat16_as_ushort(__float2bfloat16_rn(a[e]));
+            }
+        }
+        tc::cluster_sync();  // keep the cluster together until every CTA is done
     }
     tc::fence_before_sync();
     __syncthreads();
@@ -476,17 +543,36 @@ cudaError_t launch_tc(const GroupGemm &p, cudaStream_t st)
     } else if (!encode_kmajor(p.B, static_cast<int64_t>(p.G) * p.N, p.K, BN, &mb)) {  // [G N rows][K columns]
         return cudaErrorInvalidValue;
     }
+    const int rt = rblk * p.hpg;
+    const int mtiles = (p.M + rt - 1) / rt, ntiles = (p.N + BN - 1) / BN;
+    // Split K over a cluster when the tiles are short (<= 64 rows: a small
+    // batch), K is deep (>= 8 chunks) and the tiles alone would leave most SMs
+    // idle: up to 4 ways, at least two chunks each, with a ring of at most 4
+    // stages so that two CTAs share an SM and the split grid runs in one wave.
+    const int nk = (p.K + 63) / 64;
+    const int64_t tiles = static_cast<int64_t>(mtiles) * ntiles * p.G;
+    int ks = 1;
+    if (rt <= 64 && nk >= 8)
+        while (ks < 4 && tiles * ks * 2 <= (AF32 ? 152 : 2 * 152) && nk >= 4 * ks) ks *= 2;  // fp32 A: one CTA per SM
     size_t smem = 0;
     GroupGemm q = p;
-    q.stages = ring_stages<BN, AF32>(p.K, &smem);
+    q.stages = ring_stages<BN, AF32>((nk + ks - 1) / ks * 64, &smem);
+    if (ks > 1 && q.stages > 4) {
+        q.stages = 4;
+        smem = 1024 + 4 * (128 * 128 + BN * 128 + (AF32 ? 2 * 128 * 128 : 0));
+    }
     q.rblk = rblk;
+    q.ksplit = ks;
+    if (ks > 1) {  // the partials received from the cluster reuse the ring
+        const size_t need = 1024 + static_cast<size_t>(ks) * rt * (BN / ks + 4) * 4;
+        if (smem < need) smem = need;
+    }
     e = cudaFuncSetAttribute(gemm_tc_kernel<BN, NMAJ, AF32, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    const int rt = rblk * p.hpg;
-    dim3 grid((p.M + rt - 1) / rt, (p.N + BN - 1) / BN, p.G);
+    dim3 grid(mtiles * ks, ntiles, p.G);
     ProjEpi none{};
-    return launch_dependent(gemm_tc_kernel<BN, NMAJ, AF32, false>, grid, dim3(kGemmThreads), smem, st, 1, q, ma, mb,
+    return launch_dependent(gemm_tc_kernel<BN, NMAJ, AF32, false>, grid, dim3(kGemmThreads), smem, st, ks, q, ma, mb,
                             mb, mb, none);
 }
 
@@ -542,6 +628,7 @@ cudaError_t launch_proj(const mla_dims &d, const CacheView &c, int batch, int n_
     size_t smem = 0;
     p.stages = ring_stages<BN, false>(p.K, &smem);
     p.rblk = rblk;
+    p.ksplit = 1;
     e = cudaFuncSetAttribute(gemm_tc_kernel<BN, false, false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(smem));
     if (e != cudaSuccess) return e;

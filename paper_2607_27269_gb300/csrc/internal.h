@@ -74,7 +74,7 @@ struct GroupGemm {
     void *C;
     int64_t ldc;
     unsigned *status;
-    int stages, rblk;  // set by the launcher
+    int stages, rblk, ksplit;  // set by the launcher
 };
 cudaError_t launch_group_gemm(const GroupGemm &p, cudaStream_t st);
 
