@@ -444,3 +444,44 @@ int orc_project_append(const orc_dims *d, const orc_cache *c, int batch, int n_n
     }
     return err;
 }
+
+/* Acceptance statistics of a draft against its target at the same contexts
+ * (Sec. 3.3, Eqs. 9-10), one row per context, over the vocabulary:
+ *   p_D = softmax(draft row), p_T = softmax(target row)   (temperature 1)
+ *   alpha_sample = sum_y min(p_D(y), p_T(y))              (Eq. 9)
+ *   argmax_D, argmax_T: index of the largest logit, the lowest index among
+ *   equal maxima (the paper does not say how ties break); the decision is
+ *   taken on the logits themselves, softmax being monotone
+ *   greedy = [argmax_D == argmax_T]                        (Eq. 10)
+ * Logits are given as exact fp64 values; every sum is fp64.
+ *   draft, target [rows, vocab]; outputs [rows] (any may be NULL). */
+int orc_acceptance(int rows, int vocab, const double *draft, const double *target, double *alpha,
+                   int32_t *argmax_d, int32_t *argmax_t, int32_t *greedy)
+{
+    if (rows < 0 || vocab <= 0) return ORC_BAD_ARG;
+#pragma omp parallel for schedule(static)
+    for (int r = 0; r < rows; ++r) {
+        const double *d = draft + (int64_t)r * vocab, *t = target + (int64_t)r * vocab;
+        int ad = 0, at = 0;
+        for (int y = 1; y < vocab; ++y) {
+            if (d[y] > d[ad]) ad = y;
+            if (t[y] > t[at]) at = y;
+        }
+        const double md = d[ad], mt = t[at];
+        double zd = 0.0, zt = 0.0;
+        for (int y = 0; y < vocab; ++y) {
+            zd += exp(d[y] - md);
+            zt += exp(t[y] - mt);
+        }
+        double acc = 0.0;
+        for (int y = 0; y < vocab; ++y) {
+            const double pd = exp(d[y] - md) / zd, pt = exp(t[y] - mt) / zt;
+            acc += pd < pt ? pd : pt;
+        }
+        if (alpha) alpha[r] = acc;
+        if (argmax_d) argmax_d[r] = ad;
+        if (argmax_t) argmax_t[r] = at;
+        if (greedy) greedy[r] = ad == at;
+    }
+    return ORC_OK;
+}

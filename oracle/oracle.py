@@ -118,6 +118,8 @@ def configure(lib):
     lib.orc_project_append.restype = ctypes.c_int
     lib.orc_project_append.argtypes = [ctypes.POINTER(_Dims), ctypes.POINTER(_Cache), ctypes.c_int, ctypes.c_int,
                                        vp, vp, vp, vp, vp, vp, vp]
+    lib.orc_acceptance.restype = ctypes.c_int
+    lib.orc_acceptance.argtypes = [ctypes.c_int, ctypes.c_int, vp, vp, vp, vp, vp, vp]
     lib.orc_mla_decode.restype = ctypes.c_int
     lib.orc_mla_decode.argtypes = [ctypes.POINTER(_Dims), ctypes.POINTER(_Cache), ctypes.c_int,
                                    ctypes.c_int, vp, vp, vp, vp, vp, vp, vp, ctypes.c_int,
@@ -285,3 +287,20 @@ def mla_decode(dims: Dims, cache: Cache, q_nope: np.ndarray, q_pe: np.ndarray, k
     if out is not None:
         res["out"] = out
     return res
+
+
+def acceptance(draft: np.ndarray, target: np.ndarray) -> dict:
+    """Acceptance statistics of draft against target logits [rows, vocab]
+    (Sec. 3.3: Eq. 9 alpha_sample = sum_y min(p_D, p_T), Eq. 10 greedy
+    agreement of the argmaxes, lowest index on ties).  Logits are taken as
+    given (fp64)."""
+    draft = np.ascontiguousarray(draft, dtype=np.float64)
+    target = np.ascontiguousarray(target, dtype=np.float64)
+    rows, vocab = draft.shape
+    alpha = np.zeros(rows)
+    ad = np.zeros(rows, dtype=np.int32)
+    at = np.zeros(rows, dtype=np.int32)
+    gr = np.zeros(rows, dtype=np.int32)
+    _check(_load().orc_acceptance(rows, vocab, draft.ctypes.data, target.ctypes.data, alpha.ctypes.data,
+                                  ad.ctypes.data, at.ctypes.data, gr.ctypes.data), "acceptance")
+    return {"alpha_sample": alpha, "argmax_draft": ad, "argmax_target": at, "greedy": gr}

@@ -23,6 +23,12 @@ Recipe (one ``torch.Generator('cpu')`` seeded with ``seed``, drawn in this order
      ~ N(0, 1) (kr_new not yet rotated).
 Every tensor is drawn in fp32 and rounded to bf16.
 
+Draft and target logits for the acceptance statistics (``logits``) come from a
+third generator seeded with ``seed + 104729``: target rows ~ N(0, 3^2) over the
+vocabulary of the model the shape follows (a peaked distribution: the largest
+of ~10^5 draws sits ~4.5 sigma out), draft = target + N(0, 1) (a draft that
+mostly agrees), both rounded to bf16; one row per (sequence, query position).
+
 Inputs of the projection that precedes the step (``projection``) come from a
 second generator seeded with ``seed + 7919``, drawn in this order: hidden
 states h [B, q, D] ~ N(0, 1); W^DKV [r, D], W^KR [d_rope, D] and
@@ -215,3 +221,32 @@ def projection(w: Workload, seed: int = 0, hidden: Optional[int] = None) -> Proj
     w_kr = _randn(gen, (s.d_rope, D), std)
     w_q = _randn(gen, (s.num_heads * (s.d_nope + s.d_rope), D), std)
     return Projection(D, h, w_dkv, w_kr, w_q)
+
+
+# Vocabulary of the model each shape follows (Qwen2.5, Llama-3.2; the tiny
+# layer gets a small one).
+VOCAB = {
+    "tiny_b1_h8_r128_t256": 32000,
+    "qwen05b_b16_h14_r256_t2048": 151936,
+    "llama1b_chunk5_b32_h32_r512_t4096": 128256,
+    "llama3b_long_b8_h24_r512_t16k_32k": 128256,
+    "llama1b_paged_b128_h32_r512_t128_8192": 128256,
+}
+
+
+@dataclass
+class Logits:
+    draft: torch.Tensor           # bf16 [rows, vocab]
+    target: torch.Tensor          # bf16 [rows, vocab]
+
+
+def logits(name: str, seed: int = 0, rows: Optional[int] = None, vocab: Optional[int] = None) -> Logits:
+    """Draft / target logits for shape ``name``: rows = batch * q_len unless given."""
+    s = SHAPES[name]
+    R = s.batch * s.q_len if rows is None else rows
+    V = VOCAB[name] if vocab is None else vocab
+    gen = torch.Generator(device="cpu")
+    gen.manual_seed(seed + 104729)
+    t = torch.randn(R, V, generator=gen, dtype=torch.float32) * 3.0
+    d = t + torch.randn(R, V, generator=gen, dtype=torch.float32)
+    return Logits(d.to(torch.bfloat16), t.to(torch.bfloat16))

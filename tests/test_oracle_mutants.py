@@ -35,6 +35,9 @@ MUTANTS = {
                                 "orc_rope(kr, kr, dr, 0, d->rope_base, d->rope_style);\n        for (int e = 0; e < dr; ++e) c->k_rope"),
     "query_rows_head_interleaved": ("const uint16_t *w = w_q + ((int64_t)hd * dq + e) * D;",
                                     "const uint16_t *w = w_q + ((int64_t)e * H + hd) * D;"),
+    "acceptance_max_for_min": ("acc += pd < pt ? pd : pt;", "acc += pd > pt ? pd : pt;"),
+    "acceptance_target_normaliser": ("pt = exp(t[y] - mt) / zt;", "pt = exp(t[y] - mt) / zd;"),
+    "argmax_last_of_ties": ("if (d[y] > d[ad]) ad = y;", "if (d[y] >= d[ad]) ad = y;"),
     "output_projection_index": ("acc += orc_bf16_value(w[h * dv + e]) * o[(row0 + h) * dv + e];",
                                 "acc += orc_bf16_value(w[e * H + h]) * o[(row0 + h) * dv + e];"),
 }

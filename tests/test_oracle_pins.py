@@ -516,3 +516,62 @@ def test_projection_paged_equals_contiguous_and_errors():
     with pytest.raises(orc.OracleError, match="bad position"):
         orc.project_append(dims, oracle_cache(wp), bits(p.h), bits(p.w_dkv), bits(p.w_kr), None,
                            np.full(s.batch, wp.capacity, dtype=np.int32))
+
+
+# ---------------------------------------------------------------- acceptance statistics (Sec. 3.3, Eqs. 9-10)
+
+def _logits(rows, vocab, scale=3.0, seed=0):
+    g = np.random.default_rng(seed)
+    return g.standard_normal((rows, vocab)) * scale
+
+
+def test_acceptance_identical_rows():
+    d = _logits(4, 500)
+    res = orc.acceptance(d, d)
+    np.testing.assert_allclose(res["alpha_sample"], 1.0, rtol=0, atol=1e-12)
+    assert np.array_equal(res["argmax_draft"], np.argmax(d, axis=1))
+    assert np.all(res["greedy"] == 1)
+
+
+def test_acceptance_is_one_minus_total_variation():
+    """Eq. 9 states both forms: sum_y min(p_D, p_T) = 1 - TV(p_D, p_T)."""
+    d = _logits(6, 3000, seed=1)
+    t = d + 0.7 * _logits(6, 3000, scale=1.0, seed=2)
+    res = orc.acceptance(d, t)
+    pd, pt = scipy.special.softmax(d, axis=1), scipy.special.softmax(t, axis=1)
+    tv = 0.5 * np.abs(pd - pt).sum(axis=1)
+    np.testing.assert_allclose(res["alpha_sample"], 1.0 - tv, rtol=0, atol=1e-12)
+    assert np.array_equal(res["argmax_draft"], np.argmax(d, axis=1))    # numpy: first maximum
+    assert np.array_equal(res["argmax_target"], np.argmax(t, axis=1))
+    assert np.array_equal(res["greedy"], (np.argmax(d, axis=1) == np.argmax(t, axis=1)).astype(np.int32))
+    assert np.all((res["alpha_sample"] > 0) & (res["alpha_sample"] < 1))
+
+
+def test_acceptance_two_token_closed_form():
+    """Two tokens: alpha = 1 - |sigmoid(a - b) - sigmoid(c - e)|."""
+    d = np.array([[0.3, -1.2], [2.0, 2.0], [5.0, -5.0]])
+    t = np.array([[-0.4, 0.1], [2.0, 1.0], [-5.0, 5.0]])
+    res = orc.acceptance(d, t)
+    sig = lambda x: 1.0 / (1.0 + np.exp(-x))
+    ref = 1.0 - np.abs(sig(d[:, 0] - d[:, 1]) - sig(t[:, 0] - t[:, 1]))
+    np.testing.assert_allclose(res["alpha_sample"], ref, rtol=0, atol=1e-14)
+    assert list(res["argmax_draft"]) == [0, 0, 0] and list(res["argmax_target"]) == [1, 0, 1]
+    assert list(res["greedy"]) == [0, 1, 0]
+
+
+def test_acceptance_invariances_and_ties():
+    """Shifting a row's logits changes nothing; alpha is symmetric in the two
+    distributions; equal maxima resolve to the lowest index."""
+    d = _logits(5, 777, seed=3)
+    t = d + _logits(5, 777, scale=0.5, seed=4)
+    base = orc.acceptance(d, t)
+    shifted = orc.acceptance(d + 11.0, t - 3.5)
+    np.testing.assert_allclose(shifted["alpha_sample"], base["alpha_sample"], rtol=0, atol=1e-12)
+    assert np.array_equal(shifted["argmax_draft"], base["argmax_draft"])
+    swapped = orc.acceptance(t, d)
+    np.testing.assert_allclose(swapped["alpha_sample"], base["alpha_sample"], rtol=0, atol=1e-12)
+    tie = np.zeros((2, 10))
+    tie[0, [3, 7]] = 4.0
+    tie[1, [9, 2, 5]] = 1.0
+    res = orc.acceptance(tie, tie[::-1])
+    assert list(res["argmax_draft"]) == [3, 2] and list(res["argmax_target"]) == [2, 3]
