@@ -249,6 +249,7 @@ def run_ours(args, rank, world, local):
         attn_ms = [a.elapsed_time(b) / n_attn for a, b in attn_ms]
 
         proj = measure_projection(args, w, dws, stream, dev, l2, peaks=load_peaks())
+        accept = measure_acceptance(args, stream, dev, l2, peaks=load_peaks())
 
         # ---- end to end through the public API with host buffers: the step's
         # inputs (queries, new entries, lengths, positions) packed in one pinned
@@ -338,8 +339,56 @@ def run_ours(args, rank, world, local):
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": launches_per_step * args.steps,
         "project_append": proj,
+        "acceptance_stats": accept,
     }
     return line, w
+
+
+def measure_acceptance(args, stream, dev, l2, peaks):
+    """Acceptance statistics (mla_acceptance_stats) of draft against target
+    logits for every (sequence, query position) of the workload, over the
+    vocabulary of the model the shape follows, timed alone: a CUDA graph of
+    back-to-back launches over enough logits replicas that the bytes between
+    two reuses exceed 2x L2.  Algorithmic bytes: one read of both logits."""
+    import torch
+    from paper_2607_27269_gb300 import abi
+    from paper_2607_27269_gb300 import workloads as wl
+
+    lg = wl.logits(args.workload, seed=args.seed)
+    rows, vocab = lg.draft.shape
+    nbytes = 2 * lg.draft.numel() * lg.draft.element_size()
+    reps = max(2, math.ceil(2 * l2 / nbytes) + 1)
+    pairs = [(lg.draft.to(dev), lg.target.to(dev)) for _ in range(reps)]
+    outs = [torch.empty(rows, dtype=torch.float32, device=dev)] + [
+        torch.empty(rows, dtype=torch.int32, device=dev) for _ in range(3)]
+    n_launch = max(reps, 16)
+
+    def launch(i):
+        d, t = pairs[i % reps]
+        abi.acceptance_stats(d, t, *outs, stream=stream)
+
+    for i in range(3):
+        launch(i)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for i in range(n_launch):
+            launch(i)
+    g.replay()
+    torch.cuda.synchronize(dev)
+    times = []
+    for _ in range(5):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        g.replay()
+        b.record(stream)
+        times.append((a, b))
+    torch.cuda.synchronize(dev)
+    us = sum(a.elapsed_time(b) for a, b in times) / len(times) / n_launch * 1e3
+    gbs = nbytes / (us * 1e-6) / 1e9
+    return {"kernel": "mla_acceptance_stats", "us_per_launch": round(us, 3), "rows": rows, "vocab": vocab,
+            "dtype": "bf16", "bytes_per_launch": nbytes, "achieved_gbs": round(gbs, 1), "bound": "hbm",
+            "frac": round(gbs / peaks["hbm_gbs"], 4), "replicas": reps, "peak_source": peaks["source"],
+            "mean_alpha_sample": round(float(outs[0].float().mean()), 4)}
 
 
 def measure_projection(args, w, dws, stream, dev, l2, peaks):

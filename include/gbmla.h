@@ -206,6 +206,24 @@ mla_status mla_combine(const mla_dims *dims, int32_t batch, int32_t q_len, int32
 mla_status mla_out_proj(const mla_dims *dims, int32_t batch, int32_t q_len, const float *o_lat,
                         const void *w_uv, const void *w_o, void *o, void *out, void *stream);
 
+/* Acceptance statistics of a draft against its target at the same contexts
+ * (Sec. 3.3), one row per context over a vocabulary of `vocab` tokens:
+ *   p_D = softmax(draft row), p_T = softmax(target row)        (temperature 1)
+ *   alpha_sample[r]  = sum_y min(p_D(y), p_T(y))                (Eq. 9, = 1 - TV)
+ *   argmax_draft[r], argmax_target[r] = index of the largest logit, the lowest
+ *                      index among equal maxima (decided on the logits)
+ *   greedy_accept[r] = argmax_draft[r] == argmax_target[r]      (Eq. 10)
+ * draft_logits / target_logits [rows, row_stride] (the first `vocab` entries of
+ * each row used), fp32 (logits_dtype 0) or bf16 (1); both 16-byte aligned,
+ * row_stride >= vocab and row_stride * element size a multiple of 16 bytes.
+ * All arithmetic fp32.  Outputs [rows] device arrays; any may be NULL.
+ * rows == 0: no-op.  The paper has no kernel for this; it reports the two
+ * quantities its Eqs. 9-10 define. */
+mla_status mla_acceptance_stats(int32_t rows, int32_t vocab, int32_t logits_dtype, const void *draft_logits,
+                                const void *target_logits, int64_t row_stride, float *alpha_sample,
+                                int32_t *argmax_draft, int32_t *argmax_target, int32_t *greedy_accept,
+                                void *stream);
+
 /* mla_decode_attn followed by mla_combine, for callers that cannot allocate
  * device memory: code that runs where an allocation is not allowed (inside a
  * runtime that owns all device memory through its own pool, in an inference

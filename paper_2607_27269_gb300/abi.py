@@ -19,7 +19,7 @@ from . import build as _build
 
 MLA_OK, MLA_ERR_INVALID_ARG, MLA_ERR_UNSUPPORTED, MLA_ERR_CUDA, MLA_ERR_DEVICE_BOUNDS, MLA_ERR_DEVICE_TIMEOUT = range(6)
 SPLIT_TILE = 128
-EXPORTS = ("mla_workspace_size", "mla_cache_append", "mla_project_append", "mla_absorb_q", "mla_decode_attn", "mla_combine",
+EXPORTS = ("mla_workspace_size", "mla_cache_append", "mla_project_append", "mla_acceptance_stats", "mla_absorb_q", "mla_decode_attn", "mla_combine",
            "mla_out_proj", "mla_check_status", "mla_selftest_wait_timeout", "mla_decode_attn_noalloc",
            "mla_status_str", "mla_last_error")
 
@@ -71,6 +71,7 @@ def lib(auto_build: bool = True):
             L.mla_cache_append.argtypes = [P(MlaDims), P(MlaCache), i32, i32, vp, vp, vp, vp]
             L.mla_project_append.argtypes = [P(MlaDims), P(MlaCache), i32, i32, vp, vp, vp, vp, vp, vp, vp, vp]
             L.mla_absorb_q.argtypes = [P(MlaDims), i32, i32, vp, vp, vp, vp, vp, vp]
+            L.mla_acceptance_stats.argtypes = [i32, i32, i32, vp, vp, i64, vp, vp, vp, vp, vp]
             L.mla_decode_attn.argtypes = [P(MlaDims), P(MlaCache), i32, i32, vp, i32, vp, i32, vp, vp, vp]
             L.mla_combine.argtypes = [P(MlaDims), i32, i32, i32, vp, i32, vp, vp, vp, vp, vp]
             L.mla_out_proj.argtypes = [P(MlaDims), i32, i32, vp, vp, vp, vp, vp, vp]
@@ -178,6 +179,31 @@ def project_append(dims: Dims, cache: Cache, h: torch.Tensor, w_dkv: torch.Tenso
     _check("mla_project_append", lib().mla_project_append(ctypes.byref(dims.c()), ctypes.byref(cache.c()), batch,
                                                           n_new, _p(h), _p(w_dkv), _p(w_kr), _p(w_q),
                                                           _p(start_pos), _p(q_nope), _p(q_pe), _stream(stream)))
+
+
+def acceptance_stats(draft: torch.Tensor, target: torch.Tensor, alpha: Optional[torch.Tensor] = None,
+                     argmax_draft: Optional[torch.Tensor] = None, argmax_target: Optional[torch.Tensor] = None,
+                     greedy: Optional[torch.Tensor] = None, stream=None):
+    """draft / target logits [rows, vocab] (fp32 or bf16, same dtype) -> the
+    per-row overlap alpha_sample (fp32), the two argmaxes and greedy agreement
+    (int32), written into the given device tensors (allocated if None)."""
+    if draft.dtype != target.dtype or draft.dtype not in (torch.float32, torch.bfloat16) or draft.shape != target.shape:
+        raise ValueError("draft and target logits must share a shape and be fp32 or bf16")
+    rows, vocab = draft.shape
+    if draft.stride() != target.stride() or draft.stride(1) != 1 or not draft.is_cuda or not target.is_cuda:
+        raise ValueError("logits must be CUDA tensors with unit inner stride and equal row strides")
+    row_stride = draft.stride(0) if rows > 1 else vocab
+    dev = draft.device
+    alpha = torch.empty(rows, dtype=torch.float32, device=dev) if alpha is None else alpha
+    argmax_draft = torch.empty(rows, dtype=torch.int32, device=dev) if argmax_draft is None else argmax_draft
+    argmax_target = torch.empty(rows, dtype=torch.int32, device=dev) if argmax_target is None else argmax_target
+    greedy = torch.empty(rows, dtype=torch.int32, device=dev) if greedy is None else greedy
+    _check("mla_acceptance_stats", lib().mla_acceptance_stats(rows, vocab, 0 if draft.dtype == torch.float32 else 1,
+                                                              draft.data_ptr(), target.data_ptr(), row_stride,
+                                                              _p(alpha),
+                                                              _p(argmax_draft), _p(argmax_target), _p(greedy),
+                                                              _stream(stream)))
+    return alpha, argmax_draft, argmax_target, greedy
 
 
 def absorb_q(dims: Dims, q_nope: torch.Tensor, q_pe: torch.Tensor, kv_len: torch.Tensor, w_uk: torch.Tensor,

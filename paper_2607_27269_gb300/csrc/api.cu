@@ -247,6 +247,25 @@ mla_status mla_project_append(const mla_dims *dims, const mla_cache *cache, int3
                                     static_cast<cudaStream_t>(stream)));
 }
 
+mla_status mla_acceptance_stats(int32_t rows, int32_t vocab, int32_t logits_dtype, const void *draft_logits,
+                                const void *target_logits, int64_t row_stride, float *alpha_sample,
+                                int32_t *argmax_draft, int32_t *argmax_target, int32_t *greedy_accept, void *stream)
+{
+    if (rows < 0 || rows > 65535 || vocab <= 0 || row_stride < vocab) return MLA_ERR_INVALID_ARG;
+    if (logits_dtype != 0 && logits_dtype != 1) return MLA_ERR_INVALID_ARG;
+    if (rows == 0) return MLA_OK;
+    const int64_t es = logits_dtype == 0 ? 4 : 2;
+    if (!draft_logits || !target_logits || !aligned16(draft_logits) || !aligned16(target_logits) ||
+        (row_stride * es) % 16)
+        return MLA_ERR_INVALID_ARG;
+    unsigned *status = nullptr;
+    mla_status s = device_info(&status, nullptr);
+    if (s != MLA_OK) return s;
+    return from_cuda(launch_acceptance(rows, vocab, logits_dtype, draft_logits, target_logits, row_stride,
+                                       alpha_sample, argmax_draft, argmax_target, greedy_accept, status,
+                                       static_cast<cudaStream_t>(stream)));
+}
+
 mla_status mla_absorb_q(const mla_dims *dims, int32_t batch, int32_t q_len, const void *q_nope, const void *q_pe,
                         const int32_t *kv_len, const void *w_uk, void *q_abs, void *stream)
 {

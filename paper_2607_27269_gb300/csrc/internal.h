@@ -86,6 +86,11 @@ cudaError_t launch_project(const mla_dims &d, const CacheView &c, int batch, int
                            const void *w_dkv, const void *w_kr, const void *w_q, const int32_t *start_pos,
                            void *q_nope, void *q_pe, unsigned *status, cudaStream_t st);
 
+// Acceptance statistics (mla_acceptance_stats): dtype 0 = fp32, 1 = bf16 logits.
+cudaError_t launch_acceptance(int rows, int vocab, int dtype, const void *draft, const void *target, int64_t stride,
+                              float *alpha, int32_t *argmax_d, int32_t *argmax_t, int32_t *greedy, unsigned *status,
+                              cudaStream_t st);
+
 cudaError_t launch_selftest_wait(int64_t limit_ns, unsigned *status, cudaStream_t st);
 
 }  // namespace gbmla

@@ -116,3 +116,13 @@ def test_projection_arguments_are_checked_on_the_host():
     # an empty batch is a no-op
     assert L.mla_project_append(ctypes.byref(d), ctypes.byref(c), 0, 1, None, None, None, None, None, None, None,
                                 None) == abi.MLA_OK
+
+
+def test_acceptance_arguments_are_checked_on_the_host():
+    L = abi.lib()
+    assert L.mla_acceptance_stats(4, 0, 1, 16, 16, 16, None, None, None, None, None) == abi.MLA_ERR_INVALID_ARG
+    assert L.mla_acceptance_stats(4, 100, 2, 16, 16, 104, None, None, None, None, None) == abi.MLA_ERR_INVALID_ARG
+    assert L.mla_acceptance_stats(4, 100, 1, 16, 16, 99, None, None, None, None, None) == abi.MLA_ERR_INVALID_ARG
+    assert L.mla_acceptance_stats(4, 100, 1, 16, 16, 100, None, None, None, None, None) == abi.MLA_ERR_INVALID_ARG
+    assert L.mla_acceptance_stats(4, 100, 1, 24, 16, 104, None, None, None, None, None) == abi.MLA_ERR_INVALID_ARG
+    assert L.mla_acceptance_stats(0, 100, 1, None, None, 104, None, None, None, None, None) == abi.MLA_OK
