@@ -50,6 +50,10 @@ def parse_args(argv=None):
     p.add_argument("--seed", type=int, default=0)
     p.add_argument("--attn-launches", type=int, default=0,
                    help="profiling aid: one full step, then this many attention launches alone; no timing")
+    p.add_argument("--proj-launches", type=int, default=0,
+                   help="profiling aid: this many launches of the projection (mla_project_append) alone; no timing")
+    p.add_argument("--accept-launches", type=int, default=0,
+                   help="profiling aid: this many launches of the acceptance statistics alone; no timing")
     return p.parse_args(argv)
 
 
@@ -485,6 +489,40 @@ def load_peaks():
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "source": "fallback"}
 
 
+def run_kernel_only(args, local):
+    """Profiling aid (for ncu captures of one kernel on one copy of the
+    workload): `--proj-launches` launches of the projection or
+    `--accept-launches` launches of the acceptance statistics, alone.  Prints
+    one JSON line with the device status."""
+    import torch
+    from paper_2607_27269_gb300 import abi
+    from paper_2607_27269_gb300 import workloads as wl
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    w = wl.make(wl.SHAPES[args.workload], seed=args.seed)
+    if args.proj_launches > 0:
+        s = w.shape
+        p = wl.projection(w, seed=args.seed)
+        dw = abi.to_device(w, dev)
+        dims = abi.Dims(s.num_heads, s.num_kv_groups, s.d_nope, s.d_rope, s.d_v, s.rank, p.hidden, s.sm_scale,
+                        s.rope_style, s.rope_base)
+        h, a, b, c = p.h.to(dev), p.w_dkv.to(dev), p.w_kr.to(dev), p.w_q.to(dev)
+        qn, qp = torch.empty_like(dw.q_nope), torch.empty_like(dw.q_pe)
+        for _ in range(args.proj_launches):
+            abi.project_append(dims, dw.cache, h, a, b, c, dw.start_pos, qn, qp)
+        kind, n = "project_append_only", args.proj_launches
+    else:
+        lg = wl.logits(args.workload, seed=args.seed)
+        d, t = lg.draft.to(dev), lg.target.to(dev)
+        for _ in range(args.accept_launches):
+            abi.acceptance_stats(d, t)
+        kind, n = "acceptance_only", args.accept_launches
+    torch.cuda.synchronize(dev)
+    code = abi.check_status()
+    return {"profile": kind, "workload": w.shape.name, "launches": n, "status": abi.status_name(code)}, code
+
+
 def run_attn_only(args, local):
     """Profiling aid (for ncu captures of one kernel on one copy of the
     workload): one full decode step, then `--attn-launches` launches of the
@@ -605,6 +643,10 @@ def main(argv=None):
             dist.init_process_group("nccl")
     if args.attn_launches > 0:
         line, code = run_attn_only(args, local)
+        print(json.dumps(line), flush=True)
+        return 0 if code == 0 else 1
+    if args.proj_launches > 0 or args.accept_launches > 0:
+        line, code = run_kernel_only(args, local)
         print(json.dumps(line), flush=True)
         return 0 if code == 0 else 1
     if args.impl == "reference":
