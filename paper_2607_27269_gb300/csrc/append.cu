@@ -16,8 +16,9 @@ __global__ void __launch_bounds__(128) cache_append_kernel(CacheView c, int rank
                                                           const int32_t *__restrict__ start_pos,
                                                           unsigned *status)
 {
+    // no early trigger: a cache writer lets its dependents launch only once it
+    // has completed (the attention kernel loads cache tiles before its wait)
     griddep_wait();
-    griddep_launch_dependents();
     const int k = blockIdx.x, b = blockIdx.y;
     const int64_t pos = static_cast<int64_t>(start_pos[b]) + k;
     if (pos < 0 || pos >= c.capacity) {

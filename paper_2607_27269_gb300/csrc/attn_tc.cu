@@ -637,7 +637,15 @@ __global__ void __maxnreg__(128)
     __syncthreads();
     if (CL > 1) tc::cluster_sync();  // peers may multicast into this CTA only after its barriers exist
     tc::fence_after_sync();
-    griddep_wait();  // the queries and the cache entries come from the previous launches
+    // The queries come from the previous launch; the cache does not: every
+    // kernel of this library that writes the cache (append, projection) lets
+    // its dependents launch only once it has completed, so by the time this
+    // kernel runs (launched by its predecessor's trigger, which follows the
+    // predecessor's own wait) the cache is final.  So no thread waits here:
+    // the TMA producers load cache tiles at once, the query lanes wait before
+    // the first query load and the softmax warps before they write partials
+    // (a predecessor may still read the partial buffers); the MMA warps touch
+    // only shared and tensor memory.
     griddep_launch_dependents();
 
     if (part == 0 && group == 0) {
@@ -689,6 +697,8 @@ __global__ void __maxnreg__(128)
             bool has = (kind == kQK || kind == kPV) ? c < total : kind == kQuery;
             bool ok = true;
             uint64_t wait_t0 = 0;
+            bool q_pending = kind == kQuery;  // griddepcontrol.wait still to do before the first query load
+            bool first_pass = true;           // the ring lanes issue their first cache loads in it
             const uint64_t pol_keep = tc::policy_evict_last(), pol_drop = tc::policy_evict_first();
             uint32_t wbar = 0, fbar = 0, dst = 0;
             if (kind == kQK) {
@@ -709,7 +719,11 @@ __global__ void __maxnreg__(128)
                 if (!__any_sync(0xffffffffu, has && ok)) break;
                 if (any_abort()) break;
                 bool progressed = false;
-                if (has && ok) {
+                if (q_pending && !first_pass) {
+                    griddep_wait();
+                    q_pending = false;
+                }
+                if (has && ok && !q_pending) {
                     const bool ready = k == 0 || mbar_test(wbar, static_cast<uint32_t>((k - 1) & 1));
                     if (!ready) {
                         const uint64_t now = global_ns();
@@ -758,7 +772,9 @@ __global__ void __maxnreg__(128)
                     }
                 }
                 if (!__any_sync(0xffffffffu, progressed)) __nanosleep(32);
+                first_pass = false;
             }
+            if (q_pending) griddep_wait();  // (no query was loaded: keep the wait before leaving)
             if (!ok) {
                 record_status(a.status, kStatusTimeout);
                 ss.abort = 1;
@@ -904,6 +920,7 @@ __global__ void __maxnreg__(128)
         }
     } else {
         // ================================================================ softmax / epilogue
+        griddep_wait();  // before any partial is written (returns at once by the time S arrives)
         SmCtx c;
         c.lane = lane;
         c.tid = tid;

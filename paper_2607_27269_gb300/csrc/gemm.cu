@@ -255,7 +255,9 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
     __syncthreads();
     tc::fence_after_sync();
     griddep_wait();  // the activations come from the previous launch
-    griddep_launch_dependents();
+    // the projection writes the cache: its dependents launch only once it has
+    // completed (the attention kernel loads cache tiles before its own wait)
+    if (!PROJ) griddep_launch_dependents();
     const uint32_t tmem = tmem_base;
     auto bail = [&]() {
         record_status(p.status, kStatusTimeout);
