@@ -485,3 +485,102 @@ int orc_acceptance(int rows, int vocab, const double *draft, const double *targe
     }
     return ORC_OK;
 }
+
+/* ------------------------------------------------------------------ original GQA
+ * The unconverted draft the paper compares against (Sec. 3.1, Eqs. 1-4): each
+ * KV group g keeps its own key and value cache.  Keys are stored rotated to
+ * their own position (R_j k_j), so the score of query q at position p with key
+ * j is (R_p q) . (R_j k_j) = q^T R_pj k_j.  Cache blocks: sequence b, group g
+ * is block b * G + g (contiguous) or block-table row b * G + g (paged); in
+ * orc_cache, c_kv holds the values (d_v per token) and k_rope the keys (d_k). */
+typedef struct {
+    int32_t num_heads;     /* H                                        */
+    int32_t num_kv_groups; /* G, H % G == 0                            */
+    int32_t d_k;           /* key / query width per head (even)       */
+    int32_t d_v;           /* value width per head                    */
+    double sm_scale;       /* 1/sqrt(d_k)                             */
+    int32_t rope_style;
+    double rope_base;
+} orc_gqa_dims;
+
+/* New keys and values of every (sequence, group) at positions start_pos[b] + k:
+ * the key rotated in fp64 and rounded once to bf16, the value copied.
+ *   k_new [batch, G, n_new, d_k], v_new [batch, G, n_new, d_v] bf16 */
+int orc_gqa_append(const orc_gqa_dims *d, const orc_cache *c, int batch, int n_new, const uint16_t *k_new,
+                   const uint16_t *v_new, const int32_t *start_pos)
+{
+    const int G = d->num_kv_groups, dk = d->d_k, dv = d->d_v;
+    if (G <= 0 || dk <= 0 || (dk & 1) || dv <= 0 || batch < 0 || n_new < 0) return ORC_BAD_ARG;
+    double *tmp = (double *)malloc(sizeof(double) * (size_t)dk);
+    if (!tmp) return ORC_NO_MEMORY;
+    int err = ORC_OK;
+    for (int b = 0; b < batch && !err; ++b)
+        for (int g = 0; g < G && !err; ++g)
+            for (int k = 0; k < n_new && !err; ++k) {
+                const int64_t pos = (int64_t)start_pos[b] + k, e0 = ((int64_t)(b * G + g) * n_new + k);
+                int64_t co, ro;
+                err = tok_offsets(c, b * G + g, pos, &co, &ro);
+                if (err) break;
+                for (int e = 0; e < dv; ++e) c->c_kv[co + e] = v_new[e0 * dv + e];
+                for (int e = 0; e < dk; ++e) tmp[e] = orc_bf16_value(k_new[e0 * dk + e]);
+                orc_rope(tmp, tmp, dk, pos, d->rope_base, d->rope_style);
+                for (int e = 0; e < dk; ++e) c->k_rope[ro + e] = orc_bf16_round(tmp[e]);
+            }
+    free(tmp);
+    return err;
+}
+
+/* One decode step of GQA attention: for b, query i at p = kv_len[b] - q_len + i,
+ * head h of group g = h / (H / G):
+ *   s_j = sm_scale * (R_p q[b, i, h]) . K[b, g, j]   (j = 0 .. p)
+ *   o[b, i, h] = sum_j softmax(s)_j V[b, g, j],  lse = ln sum_j exp(s_j)
+ *   q [batch, q_len, H, d_k] bf16 (not rotated); o [batch, q_len, H, d_v], lse [batch, q_len, H] */
+int orc_gqa_decode(const orc_gqa_dims *d, const orc_cache *c, int batch, int q_len, const int32_t *kv_len,
+                   const uint16_t *q, double *o, double *lse)
+{
+    const int H = d->num_heads, G = d->num_kv_groups, dk = d->d_k, dv = d->d_v;
+    if (H <= 0 || G <= 0 || H % G || dk <= 0 || (dk & 1) || dv <= 0 || batch < 0 || q_len <= 0) return ORC_BAD_ARG;
+    const int hpg = H / G;
+    for (int b = 0; b < batch; ++b)
+        if (kv_len[b] < q_len || kv_len[b] > c->capacity) return ORC_BAD_POSITION;
+    const int64_t rows = (int64_t)batch * q_len * H;
+    int err = ORC_OK;
+#pragma omp parallel for schedule(dynamic)
+    for (int64_t row = 0; row < rows; ++row) {
+        const int h = (int)(row % H), i = (int)((row / H) % q_len), b = (int)(row / ((int64_t)H * q_len));
+        const int g = h / hpg;
+        const int64_t p = (int64_t)kv_len[b] - q_len + i;
+        double *qr = (double *)malloc(sizeof(double) * (size_t)(dk + p + 1));
+        if (!qr) {
+#pragma omp critical
+            err = ORC_NO_MEMORY;
+            continue;
+        }
+        double *s = qr + dk;
+        for (int e = 0; e < dk; ++e) qr[e] = orc_bf16_value(q[row * dk + e]);
+        orc_rope(qr, qr, dk, p, d->rope_base, d->rope_style);
+        double m = -INFINITY;
+        for (int64_t j = 0; j <= p; ++j) {
+            int64_t co, ro;
+            tok_offsets(c, b * G + g, j, &co, &ro);
+            double acc = 0.0;
+            for (int e = 0; e < dk; ++e) acc += qr[e] * orc_bf16_value(c->k_rope[ro + e]);
+            s[j] = d->sm_scale * acc;
+            if (s[j] > m) m = s[j];
+        }
+        double z = 0.0;
+        for (int64_t j = 0; j <= p; ++j) z += exp(s[j] - m);
+        for (int e = 0; e < dv; ++e) {
+            double acc = 0.0;
+            for (int64_t j = 0; j <= p; ++j) {
+                int64_t co, ro;
+                tok_offsets(c, b * G + g, j, &co, &ro);
+                acc += exp(s[j] - m) * orc_bf16_value(c->c_kv[co + e]);
+            }
+            o[row * dv + e] = acc / z;
+        }
+        if (lse) lse[row] = m + log(z);
+        free(qr);
+    }
+    return err;
+}

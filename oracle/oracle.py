@@ -64,6 +64,34 @@ class _Cache(ctypes.Structure):
     ]
 
 
+class _GqaDims(ctypes.Structure):
+    _fields_ = [
+        ("num_heads", ctypes.c_int32),
+        ("num_kv_groups", ctypes.c_int32),
+        ("d_k", ctypes.c_int32),
+        ("d_v", ctypes.c_int32),
+        ("sm_scale", ctypes.c_double),
+        ("rope_style", ctypes.c_int32),
+        ("rope_base", ctypes.c_double),
+    ]
+
+
+@dataclass
+class GqaDims:
+    """Shape of an original GQA layer (Sec. 3.1)."""
+    num_heads: int
+    num_kv_groups: int
+    d_k: int
+    d_v: int
+    sm_scale: float
+    rope_style: int = 0
+    rope_base: float = 10000.0
+
+    def _c(self) -> _GqaDims:
+        return _GqaDims(self.num_heads, self.num_kv_groups, self.d_k, self.d_v, self.sm_scale, self.rope_style,
+                        self.rope_base)
+
+
 def build(force: bool = False) -> str:
     """Compile ``mla_oracle.c`` with gcc (fp64, OpenMP, no fast-math)."""
     os.makedirs(_BUILD_DIR, exist_ok=True)
@@ -120,6 +148,12 @@ def configure(lib):
                                        vp, vp, vp, vp, vp, vp, vp]
     lib.orc_acceptance.restype = ctypes.c_int
     lib.orc_acceptance.argtypes = [ctypes.c_int, ctypes.c_int, vp, vp, vp, vp, vp, vp]
+    lib.orc_gqa_append.restype = ctypes.c_int
+    lib.orc_gqa_append.argtypes = [ctypes.POINTER(_GqaDims), ctypes.POINTER(_Cache), ctypes.c_int, ctypes.c_int,
+                                   vp, vp, vp]
+    lib.orc_gqa_decode.restype = ctypes.c_int
+    lib.orc_gqa_decode.argtypes = [ctypes.POINTER(_GqaDims), ctypes.POINTER(_Cache), ctypes.c_int, ctypes.c_int,
+                                   vp, vp, vp, vp]
     lib.orc_mla_decode.restype = ctypes.c_int
     lib.orc_mla_decode.argtypes = [ctypes.POINTER(_Dims), ctypes.POINTER(_Cache), ctypes.c_int,
                                    ctypes.c_int, vp, vp, vp, vp, vp, vp, vp, ctypes.c_int,
@@ -304,3 +338,25 @@ def acceptance(draft: np.ndarray, target: np.ndarray) -> dict:
     _check(_load().orc_acceptance(rows, vocab, draft.ctypes.data, target.ctypes.data, alpha.ctypes.data,
                                   ad.ctypes.data, at.ctypes.data, gr.ctypes.data), "acceptance")
     return {"alpha_sample": alpha, "argmax_draft": ad, "argmax_target": at, "greedy": gr}
+
+
+def gqa_append(dims: GqaDims, cache: Cache, k_new: np.ndarray, v_new: np.ndarray, start_pos) -> None:
+    """Original GQA cache append (Sec. 3.1): keys [B, G, n, d_k] rotated to
+    their positions (one bf16 rounding), values [B, G, n, d_v] copied; the
+    cache's c_kv holds values, k_rope keys, block (or table row) b * G + g."""
+    k_new, v_new, start_pos = _u16(k_new), _u16(v_new), _i32(start_pos)
+    batch, n_new = k_new.shape[0], k_new.shape[2]
+    _check(_load().orc_gqa_append(ctypes.byref(dims._c()), ctypes.byref(cache._c()), batch, n_new,
+                                  k_new.ctypes.data, v_new.ctypes.data, start_pos.ctypes.data), "gqa_append")
+
+
+def gqa_decode(dims: GqaDims, cache: Cache, q: np.ndarray, kv_len) -> dict:
+    """One decode step of the original GQA attention (Sec. 3.1 Eqs. 1-4):
+    q [B, q_len, H, d_k] (not rotated) -> o [B, q_len, H, d_v], lse [B, q_len, H]."""
+    q, kv_len = _u16(q), _i32(kv_len)
+    batch, q_len = q.shape[:2]
+    o = np.zeros((batch, q_len, dims.num_heads, dims.d_v))
+    lse = np.zeros((batch, q_len, dims.num_heads))
+    _check(_load().orc_gqa_decode(ctypes.byref(dims._c()), ctypes.byref(cache._c()), batch, q_len, kv_len.ctypes.data,
+                                  q.ctypes.data, o.ctypes.data, lse.ctypes.data), "gqa_decode")
+    return {"o": o, "lse": lse}

@@ -29,6 +29,14 @@ vocabulary of the model the shape follows (a peaked distribution: the largest
 of ~10^5 draws sits ~4.5 sigma out), draft = target + N(0, 1) (a draft that
 mostly agrees), both rounded to bf16; one row per (sequence, query position).
 
+The original GQA layer at the same shape (``gqa``: the draft before conversion,
+head width d = d_v of the shape for keys and values alike, one key and value
+cache per KV group) keeps the MLA workload's lengths, positions and page
+counts and draws from a fourth generator seeded with ``seed + 15485863``: the
+page permutation (paged), key and value caches ~ N(0, 1) (keys taken as
+already rotated), queries q [B, q_len, H, d] and this step's new keys and
+values [B, G, q_len, d] ~ N(0, 1).
+
 Inputs of the projection that precedes the step (``projection``) come from a
 second generator seeded with ``seed + 7919``, drawn in this order: hidden
 states h [B, q, D] ~ N(0, 1); W^DKV [r, D], W^KR [d_rope, D] and
@@ -250,3 +258,63 @@ def logits(name: str, seed: int = 0, rows: Optional[int] = None, vocab: Optional
     t = torch.randn(R, V, generator=gen, dtype=torch.float32) * 3.0
     d = t + torch.randn(R, V, generator=gen, dtype=torch.float32)
     return Logits(d.to(torch.bfloat16), t.to(torch.bfloat16))
+
+
+@dataclass
+class GqaWorkload:
+    """The original GQA layer at a shape: caches, queries and new entries."""
+    shape: Shape
+    num_heads: int
+    num_kv_groups: int
+    d: int                        # key and value width per head
+    kv_len: torch.Tensor          # int32 [B]
+    start_pos: torch.Tensor       # int32 [B]
+    capacity: int
+    k_cache: torch.Tensor         # bf16 [blocks, block_tokens, d] (rotated keys)
+    v_cache: torch.Tensor         # bf16 [blocks, block_tokens, d]
+    block_table: Optional[torch.Tensor]  # int32 [B * G, pages] (paged) or None
+    num_pages: int
+    q: torch.Tensor               # bf16 [B, q_len, H, d]
+    k_new: torch.Tensor           # bf16 [B, G, q_len, d] (not rotated)
+    v_new: torch.Tensor           # bf16 [B, G, q_len, d]
+
+    @property
+    def sm_scale(self) -> float:
+        return 1.0 / math.sqrt(self.d)
+
+    @property
+    def cache_bytes(self) -> int:
+        """Key and value bytes one attention step reads (every group's cache)."""
+        return int(self.kv_len.sum()) * self.num_kv_groups * 2 * self.d * 2
+
+
+def gqa(w: Workload, seed: int = 0) -> GqaWorkload:
+    """The original GQA layer for workload ``w`` (its lengths and layout)."""
+    s = w.shape
+    B, q = w.kv_len.numel(), w.q_nope.shape[1]
+    G, H, d = s.num_kv_groups, s.num_heads, s.d_v
+    gen = torch.Generator(device="cpu")
+    gen.manual_seed(seed + 15485863)
+    if s.paged:
+        ps = s.page_size
+        pages_per_seq = [(int(k) + ps - 1) // ps for k in w.kv_len]
+        max_pages = max(pages_per_seq) if B else 1
+        num_pages = G * sum(pages_per_seq)
+        perm = torch.randperm(num_pages, generator=gen)
+        bt = torch.full((B * G, max(max_pages, 1)), -1, dtype=torch.int32)
+        nxt = 0
+        for b, npg in enumerate(pages_per_seq):
+            for g in range(G):
+                bt[b * G + g, :npg] = perm[nxt:nxt + npg].to(torch.int32)
+                nxt += npg
+        blocks, block_tokens, cap = num_pages, ps, max_pages * ps
+    else:
+        bt, num_pages = None, 0
+        blocks, block_tokens, cap = B * G, w.capacity, w.capacity
+    k_cache = _randn(gen, (blocks, block_tokens, d))
+    v_cache = _randn(gen, (blocks, block_tokens, d))
+    qq = _randn(gen, (B, q, H, d))
+    k_new = _randn(gen, (B, G, q, d))
+    v_new = _randn(gen, (B, G, q, d))
+    return GqaWorkload(s, H, G, d, w.kv_len.clone(), w.start_pos.clone(), cap, k_cache, v_cache, bt, num_pages, qq,
+                       k_new, v_new)

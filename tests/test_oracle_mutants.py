@@ -38,6 +38,12 @@ MUTANTS = {
     "acceptance_max_for_min": ("acc += pd < pt ? pd : pt;", "acc += pd > pt ? pd : pt;"),
     "acceptance_target_normaliser": ("pt = exp(t[y] - mt) / zt;", "pt = exp(t[y] - mt) / zd;"),
     "argmax_last_of_ties": ("if (d[y] > d[ad]) ad = y;", "if (d[y] >= d[ad]) ad = y;"),
+    "gqa_query_not_rotated": ("orc_rope(qr, qr, dk, p, d->rope_base, d->rope_style);",
+                              "orc_rope(qr, qr, dk, 0, d->rope_base, d->rope_style);"),
+    "gqa_group_of_head": ("const int g = h / hpg;\n        const int64_t p = (int64_t)kv_len[b] - q_len + i;",
+                          "const int g = h % G;\n        const int64_t p = (int64_t)kv_len[b] - q_len + i;"),
+    "gqa_value_block": ("tok_offsets(c, b * G + g, j, &co, &ro);\n                acc += exp",
+                        "tok_offsets(c, b * G + (g + 1) % G, j, &co, &ro);\n                acc += exp"),
     "output_projection_index": ("acc += orc_bf16_value(w[h * dv + e]) * o[(row0 + h) * dv + e];",
                                 "acc += orc_bf16_value(w[e * H + h]) * o[(row0 + h) * dv + e];"),
 }

@@ -575,3 +575,58 @@ def test_acceptance_invariances_and_ties():
     tie[1, [9, 2, 5]] = 1.0
     res = orc.acceptance(tie, tie[::-1])
     assert list(res["argmax_draft"]) == [3, 2] and list(res["argmax_target"]) == [2, 3]
+
+
+# ---------------------------------------------------------------- original GQA (Sec. 3.1, Eqs. 1-4)
+
+def _gqa_case(paged, q_len=3, seed=21):
+    s = wl.Shape("gqa_test", 3, 6, 2, 8, 8, 8, 16, 0, q_len, 5, 14, paged=paged, page_size=4)
+    w = wl.make(s, seed=seed)
+    gw = wl.gqa(w, seed=seed)
+    dims = orc.GqaDims(gw.num_heads, gw.num_kv_groups, gw.d, gw.d, gw.sm_scale)
+    bt = None if gw.block_table is None else gw.block_table.numpy().astype(np.int32).copy()
+    cache = orc.Cache(c_kv=bits(gw.v_cache), k_rope=bits(gw.k_cache), c_tok_stride=gw.d, r_tok_stride=gw.d,
+                      c_blk_stride=gw.k_cache.shape[1] * gw.d, r_blk_stride=gw.k_cache.shape[1] * gw.d,
+                      capacity=gw.capacity, block_table=bt, page_size=s.page_size if paged else 0,
+                      num_pages=gw.num_pages)
+    return s, gw, dims, cache
+
+
+def _gqa_logical(gw, cache, b, g, t):
+    """(rotated key, value) of token t of sequence b, group g, read through the block table."""
+    if cache.block_table is not None:
+        blk, slot = cache.block_table[b * gw.num_kv_groups + g, t // 4], t % 4
+    else:
+        blk, slot = b * gw.num_kv_groups + g, t
+    return bf16_to_f64(cache.k_rope[blk, slot]), bf16_to_f64(cache.c_kv[blk, slot])
+
+
+@pytest.mark.parametrize("paged", [False, True])
+def test_gqa_oracle_matches_sdpa(paged):
+    """Append then decode, against torch SDPA over keys rotated by the complex
+    form and a causal chunk mask."""
+    s, gw, dims, cache = _gqa_case(paged)
+    orc.gqa_append(dims, cache, bits(gw.k_new), bits(gw.v_new), gw.start_pos.numpy())
+    res = orc.gqa_decode(dims, cache, bits(gw.q), gw.kv_len.numpy())
+    H, G, d, q_len = gw.num_heads, gw.num_kv_groups, gw.d, s.q_len
+    for b in range(s.batch):
+        kv = int(gw.kv_len[b])
+        for t in range(int(gw.start_pos[b]), kv):          # appended keys: one rounding of the exact rotation
+            for g in range(G):
+                k, _ = _gqa_logical(gw, cache, b, g, t)
+                exact = rope_complex(bf16_to_f64(bits(gw.k_new))[b, g, t - int(gw.start_pos[b])], t)
+                ulp = 2.0 ** (np.floor(np.log2(np.maximum(np.abs(exact), 1e-30))) - 7)
+                assert np.all(np.abs(k - exact) <= ulp / 2 + 1e-15)
+        K = np.stack([np.stack([_gqa_logical(gw, cache, b, g, t)[0] for t in range(kv)]) for g in range(G)])
+        V = np.stack([np.stack([_gqa_logical(gw, cache, b, g, t)[1] for t in range(kv)]) for g in range(G)])
+        pos = kv - q_len + np.arange(q_len)
+        Q = np.stack([rope_complex(bf16_to_f64(bits(gw.q))[b, i], pos[i]) for i in range(q_len)])  # [q, H, d]
+        mask = np.arange(kv)[None, :] <= pos[:, None]                                              # [q, kv]
+        qt = torch.from_numpy(Q.transpose(1, 0, 2))[None]                                         # [1, H, q, d]
+        kt = torch.from_numpy(K)[None].repeat_interleave(H // G, dim=1)
+        vt = torch.from_numpy(V)[None].repeat_interleave(H // G, dim=1)
+        ref = F.scaled_dot_product_attention(qt, kt, vt, attn_mask=torch.from_numpy(mask), scale=gw.sm_scale)
+        np.testing.assert_allclose(res["o"][b].transpose(1, 0, 2), ref[0].numpy(), rtol=1e-12, atol=1e-12)
+        logits = np.einsum("qhd,htd->hqt", Q, np.repeat(K, H // G, axis=0)) * gw.sm_scale
+        logits = np.where(mask[None], logits, -np.inf)
+        np.testing.assert_allclose(res["lse"][b].T, scipy.special.logsumexp(logits, axis=2), rtol=1e-12, atol=1e-12)
