@@ -54,6 +54,8 @@ def parse_args(argv=None):
                    help="profiling aid: this many launches of the projection (mla_project_append) alone; no timing")
     p.add_argument("--accept-launches", type=int, default=0,
                    help="profiling aid: this many launches of the acceptance statistics alone; no timing")
+    p.add_argument("--gqa-launches", type=int, default=0,
+                   help="profiling aid: this many launches of the original-GQA attention alone; no timing")
     return p.parse_args(argv)
 
 
@@ -254,6 +256,7 @@ def run_ours(args, rank, world, local):
 
         proj = measure_projection(args, w, dws, stream, dev, l2, peaks=load_peaks())
         accept = measure_acceptance(args, stream, dev, l2, peaks=load_peaks())
+        gqa = measure_gqa(args, w, dws, steps, stream, dev, l2, peaks=load_peaks())
 
         # ---- end to end through the public API with host buffers: the step's
         # inputs (queries, new entries, lengths, positions) packed in one pinned
@@ -344,8 +347,77 @@ def run_ours(args, rank, world, local):
         "gpu_launches": launches_per_step * args.steps,
         "project_append": proj,
         "acceptance_stats": accept,
+        "gqa_comparison": gqa,
     }
     return line, w
+
+
+def _graph_time_us(launch, n_launch, stream, dev):
+    import torch
+    for i in range(3):
+        launch(i)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for i in range(n_launch):
+            launch(i)
+    g.replay()
+    torch.cuda.synchronize(dev)
+    times = []
+    for _ in range(5):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        g.replay()
+        b.record(stream)
+        times.append((a, b))
+    torch.cuda.synchronize(dev)
+    return sum(a.elapsed_time(b) for a, b in times) / len(times) / n_launch * 1e3
+
+
+def measure_gqa(args, w, dws, steps, stream, dev, l2, peaks):
+    """The original GQA draft's attention at the same shape (mla_gqa_decode_attn:
+    split-KV attention and merge) beside the MLA path's (mla_decode_attn +
+    mla_combine), both as CUDA graphs of back-to-back calls over replicas
+    beyond 2x L2.  Bytes: the cache each reads per step."""
+    import torch
+    from paper_2607_27269_gb300 import abi
+    from paper_2607_27269_gb300 import workloads as wl
+
+    gw = wl.gqa(w, seed=args.seed)
+    s = w.shape
+    per = (gw.k_cache.numel() + gw.v_cache.numel()) * 2
+    reps = max(2, math.ceil(2 * l2 / per) + 1)
+    dims = abi.GqaDims(gw.num_heads, gw.num_kv_groups, gw.d, gw.sm_scale, s.rope_style, s.rope_base)
+    runs = []
+    for _ in range(reps):
+        bt = None if gw.block_table is None else gw.block_table.to(dev)
+        cache = abi.Cache(gw.v_cache.to(dev), gw.k_cache.to(dev), gw.capacity, bt, s.page_size if s.paged else 0,
+                          gw.num_pages)
+        st = abi.GqaStep(dims, cache, gw.kv_len.numel(), gw.q.shape[1], int(gw.kv_len.max()), args.num_splits)
+        runs.append((st, gw.q.to(dev), gw.kv_len.to(dev)))
+    n = max(reps, 16)
+    gqa_us = _graph_time_us(lambda i: runs[i % reps][0](runs[i % reps][1], runs[i % reps][2], stream=stream), n,
+                            stream, dev)
+    code = abi.check_status(stream)
+    if code != abi.MLA_OK:
+        raise RuntimeError(f"device status after the GQA attention: {abi.status_name(code)}")
+    R = len(dws)
+
+    def mla(i):
+        d, st = dws[i % R], steps[i % R]
+        abi.decode_attn(d.dims, d.cache, d.kv_len, d.max_kv_len, st.q_abs, st.o_part, st.lse_part, st.num_splits,
+                        stream)
+        abi.combine(d.dims, d.batch, d.q_len, d.kv_len, d.max_kv_len, st.o_part, st.lse_part, st.o_lat, st.lse,
+                    st.num_splits, stream)
+
+    mla_us = _graph_time_us(mla, max(R, 16), stream, dev)
+    gqa_bytes, mla_bytes = gw.cache_bytes, w.cache_bytes
+    gbs = gqa_bytes / (gqa_us * 1e-6) / 1e9
+    del runs
+    return {"kernel": "mla_gqa_decode_attn", "head_dim": gw.d, "gqa_us": round(gqa_us, 3),
+            "mla_us": round(mla_us, 3), "gqa_cache_bytes": gqa_bytes, "mla_cache_bytes": mla_bytes,
+            "cache_bytes_ratio_mla_over_gqa": round(mla_bytes / gqa_bytes, 4),
+            "time_ratio_mla_over_gqa": round(mla_us / gqa_us, 4), "gqa_achieved_gbs": round(gbs, 1),
+            "gqa_frac": round(gbs / peaks["hbm_gbs"], 4), "replicas": reps, "peak_source": peaks["source"]}
 
 
 def measure_acceptance(args, stream, dev, l2, peaks):
@@ -512,6 +584,18 @@ def run_kernel_only(args, local):
         for _ in range(args.proj_launches):
             abi.project_append(dims, dw.cache, h, a, b, c, dw.start_pos, qn, qp)
         kind, n = "project_append_only", args.proj_launches
+    elif args.gqa_launches > 0:
+        s = w.shape
+        gw = wl.gqa(w, seed=args.seed)
+        dims = abi.GqaDims(gw.num_heads, gw.num_kv_groups, gw.d, gw.sm_scale, s.rope_style, s.rope_base)
+        bt = None if gw.block_table is None else gw.block_table.to(dev)
+        cache = abi.Cache(gw.v_cache.to(dev), gw.k_cache.to(dev), gw.capacity, bt, s.page_size if s.paged else 0,
+                          gw.num_pages)
+        st = abi.GqaStep(dims, cache, gw.kv_len.numel(), gw.q.shape[1], int(gw.kv_len.max()), args.num_splits)
+        q, kv = gw.q.to(dev), gw.kv_len.to(dev)
+        for _ in range(args.gqa_launches):
+            st(q, kv)
+        kind, n = "gqa_attention_only", args.gqa_launches
     else:
         lg = wl.logits(args.workload, seed=args.seed)
         d, t = lg.draft.to(dev), lg.target.to(dev)
@@ -645,7 +729,7 @@ def main(argv=None):
         line, code = run_attn_only(args, local)
         print(json.dumps(line), flush=True)
         return 0 if code == 0 else 1
-    if args.proj_launches > 0 or args.accept_launches > 0:
+    if args.proj_launches > 0 or args.accept_launches > 0 or args.gqa_launches > 0:
         line, code = run_kernel_only(args, local)
         print(json.dumps(line), flush=True)
         return 0 if code == 0 else 1

@@ -224,6 +224,47 @@ mla_status mla_acceptance_stats(int32_t rows, int32_t vocab, int32_t logits_dtyp
                                 int32_t *argmax_draft, int32_t *argmax_target, int32_t *greedy_accept,
                                 void *stream);
 
+/* ---- The original GQA draft at the same shapes (Sec. 3.1, Eqs. 1-4): the
+ * model the converted MLA draft replaces, for comparing cache bytes and step
+ * time.  Each KV group g of sequence b has its own key and value cache; unit
+ * u = b*G + g addresses them through an mla_cache whose k_rope holds the keys
+ * (stored rotated to their position, head_dim per token) and c_kv the values
+ * (head_dim per token), block u (contiguous) or block-table row u (paged),
+ * with the same stride, alignment and page rules as the MLA cache. */
+typedef struct mla_gqa_dims {
+    int32_t num_heads;      /* H                                        */
+    int32_t num_kv_groups;  /* G, H % G == 0                            */
+    int32_t head_dim;       /* key = value width per head: 64 or 128    */
+    float sm_scale;         /* 1/sqrt(head_dim)                         */
+    int32_t rope_style;     /* as in mla_dims, over the whole head      */
+    float rope_base;
+} mla_gqa_dims;
+
+/* New keys and values of every (sequence, group) at positions start_pos[b] + k:
+ * keys rotated in fp32 and rounded once to bf16, values copied.
+ *   k_new, v_new [batch, G, n_new, head_dim] bf16; start_pos [batch] int32.
+ * Faults as for mla_cache_append. */
+mla_status mla_gqa_append(const mla_gqa_dims *dims, const mla_cache *cache, int32_t batch, int32_t n_new,
+                          const void *k_new, const void *v_new, const int32_t *start_pos, void *stream);
+
+/* Partial-buffer sizes and split count of mla_gqa_decode_attn (as
+ * mla_workspace_size, over the batch*G units). */
+mla_status mla_gqa_workspace_size(const mla_gqa_dims *dims, int32_t batch, int32_t q_len, int32_t max_kv_len,
+                                  int32_t num_splits, size_t *o_part_bytes, size_t *lse_part_bytes,
+                                  int32_t *num_splits_used);
+
+/* One decode step of GQA attention, split over the units' 128-token tiles and
+ * merged: for query i of sequence b at p = kv_len[b] - q_len + i and head h
+ * of group g = h / (H/G),
+ *   o = sum_j softmax_j(sm_scale (R_p q[b,i,h]) . K[b,g,j]) V[b,g,j],  j <= p
+ * q [batch, q_len, H, head_dim] bf16 (not rotated), q_len * H/G <= 128;
+ * o_part / lse_part sized by mla_gqa_workspace_size; outputs in group-major
+ * order: o [batch, G, q_len, H/G, head_dim] fp32, lse [batch, G, q_len, H/G]
+ * fp32 (natural log) or NULL. */
+mla_status mla_gqa_decode_attn(const mla_gqa_dims *dims, const mla_cache *cache, int32_t batch, int32_t q_len,
+                               const int32_t *kv_len, int32_t max_kv_len, const void *q, int32_t num_splits,
+                               float *o_part, float *lse_part, float *o, float *lse, void *stream);
+
 /* mla_decode_attn followed by mla_combine, for callers that cannot allocate
  * device memory: code that runs where an allocation is not allowed (inside a
  * runtime that owns all device memory through its own pool, in an inference

@@ -19,7 +19,8 @@ from . import build as _build
 
 MLA_OK, MLA_ERR_INVALID_ARG, MLA_ERR_UNSUPPORTED, MLA_ERR_CUDA, MLA_ERR_DEVICE_BOUNDS, MLA_ERR_DEVICE_TIMEOUT = range(6)
 SPLIT_TILE = 128
-EXPORTS = ("mla_workspace_size", "mla_cache_append", "mla_project_append", "mla_acceptance_stats", "mla_absorb_q", "mla_decode_attn", "mla_combine",
+EXPORTS = ("mla_workspace_size", "mla_cache_append", "mla_project_append", "mla_acceptance_stats",
+           "mla_gqa_append", "mla_gqa_workspace_size", "mla_gqa_decode_attn", "mla_absorb_q", "mla_decode_attn", "mla_combine",
            "mla_out_proj", "mla_check_status", "mla_selftest_wait_timeout", "mla_decode_attn_noalloc",
            "mla_status_str", "mla_last_error")
 
@@ -36,6 +37,11 @@ class MlaDims(ctypes.Structure):
                 ("d_rope", ctypes.c_int32), ("d_v", ctypes.c_int32), ("rank", ctypes.c_int32),
                 ("hidden", ctypes.c_int32), ("sm_scale", ctypes.c_float), ("rope_style", ctypes.c_int32),
                 ("rope_base", ctypes.c_float)]
+
+
+class MlaGqaDims(ctypes.Structure):
+    _fields_ = [("num_heads", ctypes.c_int32), ("num_kv_groups", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("sm_scale", ctypes.c_float), ("rope_style", ctypes.c_int32), ("rope_base", ctypes.c_float)]
 
 
 class MlaCache(ctypes.Structure):
@@ -72,6 +78,10 @@ def lib(auto_build: bool = True):
             L.mla_project_append.argtypes = [P(MlaDims), P(MlaCache), i32, i32, vp, vp, vp, vp, vp, vp, vp, vp]
             L.mla_absorb_q.argtypes = [P(MlaDims), i32, i32, vp, vp, vp, vp, vp, vp]
             L.mla_acceptance_stats.argtypes = [i32, i32, i32, vp, vp, i64, vp, vp, vp, vp, vp]
+            L.mla_gqa_append.argtypes = [P(MlaGqaDims), P(MlaCache), i32, i32, vp, vp, vp, vp]
+            L.mla_gqa_workspace_size.argtypes = [P(MlaGqaDims), i32, i32, i32, i32, P(sz), P(sz), P(i32)]
+            L.mla_gqa_decode_attn.argtypes = [P(MlaGqaDims), P(MlaCache), i32, i32, vp, i32, vp, i32, vp, vp, vp, vp,
+                                              vp]
             L.mla_decode_attn.argtypes = [P(MlaDims), P(MlaCache), i32, i32, vp, i32, vp, i32, vp, vp, vp]
             L.mla_combine.argtypes = [P(MlaDims), i32, i32, i32, vp, i32, vp, vp, vp, vp, vp]
             L.mla_out_proj.argtypes = [P(MlaDims), i32, i32, vp, vp, vp, vp, vp, vp]
@@ -179,6 +189,59 @@ def project_append(dims: Dims, cache: Cache, h: torch.Tensor, w_dkv: torch.Tenso
     _check("mla_project_append", lib().mla_project_append(ctypes.byref(dims.c()), ctypes.byref(cache.c()), batch,
                                                           n_new, _p(h), _p(w_dkv), _p(w_kr), _p(w_q),
                                                           _p(start_pos), _p(q_nope), _p(q_pe), _stream(stream)))
+
+
+@dataclass
+class GqaDims:
+    """Shape of an original GQA layer (key and value width head_dim)."""
+    num_heads: int
+    num_kv_groups: int
+    head_dim: int
+    sm_scale: float
+    rope_style: int = 0
+    rope_base: float = 10000.0
+
+    def c(self) -> MlaGqaDims:
+        return MlaGqaDims(self.num_heads, self.num_kv_groups, self.head_dim, self.sm_scale, self.rope_style,
+                          self.rope_base)
+
+
+def gqa_append(dims: GqaDims, cache: Cache, k_new: torch.Tensor, v_new: torch.Tensor, start_pos: torch.Tensor,
+               stream=None):
+    """k_new / v_new [B, G, n, head_dim] into the GQA cache (keys in cache.k_rope, values in cache.c_kv)."""
+    batch, n_new = k_new.shape[0], k_new.shape[2]
+    _check("mla_gqa_append", lib().mla_gqa_append(ctypes.byref(dims.c()), ctypes.byref(cache.c()), batch, n_new,
+                                                  _p(k_new), _p(v_new), _p(start_pos), _stream(stream)))
+
+
+def gqa_workspace_size(dims: GqaDims, batch: int, q_len: int, max_kv_len: int, num_splits: int = 0):
+    ob, lb, s = ctypes.c_size_t(), ctypes.c_size_t(), ctypes.c_int32()
+    _check("mla_gqa_workspace_size", lib().mla_gqa_workspace_size(ctypes.byref(dims.c()), batch, q_len, max_kv_len,
+                                                                  num_splits, ctypes.byref(ob), ctypes.byref(lb),
+                                                                  ctypes.byref(s)))
+    return ob.value, lb.value, s.value
+
+
+class GqaStep:
+    """GQA decode attention with its partial buffers allocated once:
+    o [B, G, q_len, H/G, head_dim] fp32 (group-major), lse [B, G, q_len, H/G]."""
+
+    def __init__(self, dims: GqaDims, cache: Cache, batch: int, q_len: int, max_kv_len: int, num_splits: int = 0):
+        self.dims, self.cache, self.batch, self.q_len, self.max_kv_len = dims, cache, batch, q_len, max_kv_len
+        dev = cache.c_kv.device
+        ob, lb, self.num_splits = gqa_workspace_size(dims, batch, q_len, max_kv_len, num_splits)
+        G, hpg, d = dims.num_kv_groups, dims.num_heads // dims.num_kv_groups, dims.head_dim
+        self.o_part = torch.empty(max(ob // 4, 1), dtype=torch.float32, device=dev)
+        self.lse_part = torch.empty(max(lb // 4, 1), dtype=torch.float32, device=dev)
+        self.o = torch.empty(batch, G, q_len, hpg, d, dtype=torch.float32, device=dev)
+        self.lse = torch.empty(batch, G, q_len, hpg, dtype=torch.float32, device=dev)
+
+    def __call__(self, q: torch.Tensor, kv_len: torch.Tensor, stream=None):
+        _check("mla_gqa_decode_attn", lib().mla_gqa_decode_attn(
+            ctypes.byref(self.dims.c()), ctypes.byref(self.cache.c()), self.batch, self.q_len, _p(kv_len),
+            self.max_kv_len, _p(q), self.num_splits, _p(self.o_part), _p(self.lse_part), _p(self.o), _p(self.lse),
+            _stream(stream)))
+        return self.o
 
 
 def acceptance_stats(draft: torch.Tensor, target: torch.Tensor, alpha: Optional[torch.Tensor] = None,

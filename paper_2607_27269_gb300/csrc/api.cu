@@ -266,6 +266,116 @@ mla_status mla_acceptance_stats(int32_t rows, int32_t vocab, int32_t logits_dtyp
                                        static_cast<cudaStream_t>(stream)));
 }
 
+// ---- original GQA
+namespace {
+// The GQA layer seen through the MLA checks: values where the latent goes,
+// keys where the positional keys go.
+mla_status gqa_as_mla(const mla_gqa_dims *g, mla_dims *d)
+{
+    if (!g || g->num_heads <= 0 || g->num_kv_groups <= 0 || g->num_heads % g->num_kv_groups)
+        return MLA_ERR_INVALID_ARG;
+    if (!(g->sm_scale > 0.f) || !isfinite(g->sm_scale) || !(g->rope_base > 1.f) || !isfinite(g->rope_base))
+        return MLA_ERR_INVALID_ARG;
+    if (g->rope_style != 0 && g->rope_style != 1) return MLA_ERR_INVALID_ARG;
+    if (g->head_dim != 64 && g->head_dim != 128) return MLA_ERR_UNSUPPORTED;
+    *d = mla_dims{g->num_heads, g->num_kv_groups, g->head_dim, g->head_dim, g->head_dim, g->head_dim, 0,
+                  g->sm_scale, g->rope_style, g->rope_base};
+    return MLA_OK;
+}
+
+int gqa_splits(const mla_gqa_dims *g, int batch, int max_kv_len, int requested, int sms)
+{
+    if (requested > 0) return requested;
+    int64_t s = sms;  // one CTA per SM
+    const int64_t tiles = static_cast<int64_t>(batch) * g->num_kv_groups * ((max_kv_len + MLA_SPLIT_TILE - 1) / MLA_SPLIT_TILE);
+    if (s > tiles) s = tiles;
+    return s < 1 ? 1 : static_cast<int>(s);
+}
+}  // namespace
+
+mla_status mla_gqa_append(const mla_gqa_dims *dims, const mla_cache *cache, int32_t batch, int32_t n_new,
+                          const void *k_new, const void *v_new, const int32_t *start_pos, void *stream)
+{
+    mla_dims d;
+    mla_status s = gqa_as_mla(dims, &d);
+    if (s != MLA_OK) return s;
+    CacheView v;
+    if ((s = check_cache(&d, cache, &v)) != MLA_OK) return s;
+    if (batch < 0 || n_new < 0 || static_cast<int64_t>(batch) * dims->num_kv_groups > 65535 || n_new > 65535)
+        return MLA_ERR_INVALID_ARG;
+    if (batch == 0 || n_new == 0) return MLA_OK;
+    if (!k_new || !v_new || !start_pos || !aligned16(v_new)) return MLA_ERR_INVALID_ARG;
+    unsigned *status = nullptr;
+    if ((s = device_info(&status, nullptr)) != MLA_OK) return s;
+    return from_cuda(launch_append(d, v, batch * dims->num_kv_groups, n_new, v_new, k_new, start_pos, status,
+                                   static_cast<cudaStream_t>(stream), dims->num_kv_groups));
+}
+
+mla_status mla_gqa_workspace_size(const mla_gqa_dims *dims, int32_t batch, int32_t q_len, int32_t max_kv_len,
+                                  int32_t num_splits, size_t *o_part_bytes, size_t *lse_part_bytes,
+                                  int32_t *num_splits_used)
+{
+    mla_dims d;
+    mla_status s = gqa_as_mla(dims, &d);
+    if (s != MLA_OK) return s;
+    if (batch < 0 || q_len < 1 || q_len > 16 || max_kv_len < q_len || num_splits < 0) return MLA_ERR_INVALID_ARG;
+    if (q_len * (dims->num_heads / dims->num_kv_groups) > 128) return MLA_ERR_UNSUPPORTED;
+    int sms = 0;
+    if ((s = device_info(nullptr, &sms)) != MLA_OK) return s;
+    const int S = gqa_splits(dims, batch, max_kv_len, num_splits, sms);
+    const size_t units = static_cast<size_t>(batch) * dims->num_kv_groups;
+    const size_t slots = units > 0 ? units + S - 1 : 0;
+    const size_t rows = static_cast<size_t>(q_len) * (dims->num_heads / dims->num_kv_groups);
+    if (o_part_bytes) *o_part_bytes = slots * rows * dims->head_dim * sizeof(float);
+    if (lse_part_bytes) *lse_part_bytes = slots * rows * sizeof(float);
+    if (num_splits_used) *num_splits_used = S;
+    return MLA_OK;
+}
+
+mla_status mla_gqa_decode_attn(const mla_gqa_dims *dims, const mla_cache *cache, int32_t batch, int32_t q_len,
+                               const int32_t *kv_len, int32_t max_kv_len, const void *q, int32_t num_splits,
+                               float *o_part, float *lse_part, float *o, float *lse, void *stream)
+{
+    mla_dims d;
+    mla_status s = gqa_as_mla(dims, &d);
+    if (s != MLA_OK) return s;
+    CacheView v;
+    if ((s = check_cache(&d, cache, &v)) != MLA_OK) return s;
+    if (batch < 0 || q_len < 1 || q_len > 16 || num_splits < 0 || num_splits > 65535) return MLA_ERR_INVALID_ARG;
+    if (static_cast<int64_t>(batch) * dims->num_kv_groups > 65535) return MLA_ERR_UNSUPPORTED;
+    if (max_kv_len < q_len || max_kv_len > cache->capacity) return MLA_ERR_INVALID_ARG;
+    const int hpg = dims->num_heads / dims->num_kv_groups;
+    if (q_len * hpg > 128) return MLA_ERR_UNSUPPORTED;
+    if (batch == 0) return MLA_OK;
+    if (!kv_len || !q || !o_part || !lse_part || !o || !aligned16(q) || !aligned16(o_part) || !aligned16(o))
+        return MLA_ERR_INVALID_ARG;
+    unsigned *status = nullptr;
+    int sms = 0;
+    if ((s = device_info(&status, &sms)) != MLA_OK) return s;
+    GqaLaunch g;
+    g.batch = batch;
+    g.q_len = q_len;
+    g.groups = dims->num_kv_groups;
+    g.hpg = hpg;
+    g.head_dim = dims->head_dim;
+    g.max_kv = max_kv_len;
+    g.num_splits = gqa_splits(dims, batch, max_kv_len, num_splits, sms);
+    g.sm_scale = dims->sm_scale;
+    g.rope_style = dims->rope_style;
+    g.rope_base = dims->rope_base;
+    g.kv_len = kv_len;
+    g.q = q;
+    g.o_part = o_part;
+    g.lse_part = lse_part;
+    g.status = status;
+    g.cache = v;
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaError_t e = launch_gqa_attn(g, st);
+    if (e != cudaSuccess) return from_cuda(e);
+    return from_cuda(launch_combine(batch * g.groups, q_len, hpg, dims->head_dim, max_kv_len, g.num_splits, kv_len,
+                                    o_part, lse_part, o, lse, st, g.groups));
+}
+
 mla_status mla_absorb_q(const mla_dims *dims, int32_t batch, int32_t q_len, const void *q_nope, const void *q_pe,
                         const int32_t *kv_len, const void *w_uk, void *q_abs, void *stream)
 {

@@ -14,13 +14,13 @@ __global__ void __launch_bounds__(128) cache_append_kernel(CacheView c, int rank
                                                           const uint16_t *__restrict__ c_new,
                                                           const uint16_t *__restrict__ kr_new,
                                                           const int32_t *__restrict__ start_pos,
-                                                          unsigned *status)
+                                                          unsigned *status, int groups)
 {
     // no early trigger: a cache writer lets its dependents launch only once it
     // has completed (the attention kernel loads cache tiles before its wait)
     griddep_wait();
     const int k = blockIdx.x, b = blockIdx.y;
-    const int64_t pos = static_cast<int64_t>(start_pos[b]) + k;
+    const int64_t pos = static_cast<int64_t>(start_pos[b / groups]) + k;
     if (pos < 0 || pos >= c.capacity) {
         if (threadIdx.x == 0) record_status(status, kStatusBounds);
         return;
@@ -62,12 +62,13 @@ __global__ void __launch_bounds__(128) cache_append_kernel(CacheView c, int rank
 }  // namespace
 
 cudaError_t launch_append(const mla_dims &d, const CacheView &c, int batch, int n_new, const void *c_new,
-                          const void *kr_new, const int32_t *start_pos, unsigned *status, cudaStream_t st)
+                          const void *kr_new, const int32_t *start_pos, unsigned *status, cudaStream_t st,
+                          int groups)
 {
     dim3 grid(n_new, batch);
     return launch_dependent(cache_append_kernel, grid, dim3(128), 0, st, 1, c, d.rank, d.d_rope, d.rope_style,
                             rope_turns(d.d_rope, d.rope_base), n_new, static_cast<const uint16_t *>(c_new),
-                            static_cast<const uint16_t *>(kr_new), start_pos, status);
+                            static_cast<const uint16_t *>(kr_new), start_pos, status, groups);
 }
 
 }  // namespace gbmla

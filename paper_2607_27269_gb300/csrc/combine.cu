@@ -23,15 +23,15 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(int batch, int
                                                                  int S, const int32_t *__restrict__ kv_len,
                                                                  const float *__restrict__ o_part,
                                                                  const float *__restrict__ lse_part, float *o_lat,
-                                                                 float *lse_out)
+                                                                 float *lse_out, int groups)
 {
     griddep_wait();
     griddep_launch_dependents();
     __shared__ int64_t red[64];
-    const int b = blockIdx.y;
+    const int b = blockIdx.y;  // unit b: sequence b / groups (groups > 1: one unit per KV group)
     int64_t T, t0;
-    block_tile_sums(kv_len, batch, b, q_len, max_kv, red, &T, &t0);
-    const int64_t nb = seq_tiles(kv_len[b], q_len, max_kv);
+    block_tile_sums(kv_len, batch, b, q_len, max_kv, red, &T, &t0, groups);
+    const int64_t nb = seq_tiles(kv_len[b / groups], q_len, max_kv);
     if (nb == 0 || T == 0) return;  // invalid length: recorded by the attention kernel
     const int k_first = part_of_tile(t0, T, S), k_last = part_of_tile(t0 + nb - 1, T, S);
     const int rows = q_len * H;
@@ -110,7 +110,7 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(int batch, int
 
 cudaError_t launch_combine(int batch, int q_len, int num_heads, int rank, int max_kv, int num_splits,
                            const int32_t *kv_len, const float *o_part, const float *lse_part, float *o_lat,
-                           float *lse, cudaStream_t st)
+                           float *lse, cudaStream_t st, int groups)
 {
     // rank is a multiple of 64 (<= 512): rank / 4 <= 128 threads per row
     const int tpr = rank / 4, rpb = kCombineThreads / tpr;
@@ -121,11 +121,11 @@ cudaError_t launch_combine(int batch, int q_len, int num_heads, int rank, int ma
     if (blocks1 >= 16 * 152) {
         dim3 grid((rows + 4 * rpb - 1) / (4 * rpb), batch);
         return launch_dependent(combine_kernel<4, 2>, grid, dim3(kCombineThreads), 0, st, 1, batch, q_len, num_heads,
-                                rank, max_kv, num_splits, kv_len, o_part, lse_part, o_lat, lse);
+                                rank, max_kv, num_splits, kv_len, o_part, lse_part, o_lat, lse, groups);
     }
     dim3 grid((rows + rpb - 1) / rpb, batch);
     return launch_dependent(combine_kernel<1, 8>, grid, dim3(kCombineThreads), 0, st, 1, batch, q_len, num_heads, rank,
-                            max_kv, num_splits, kv_len, o_part, lse_part, o_lat, lse);
+                            max_kv, num_splits, kv_len, o_part, lse_part, o_lat, lse, groups);
 }
 
 }  // namespace gbmla

@@ -140,11 +140,13 @@ __device__ __forceinline__ int64_t seq_tiles(int kv, int q_len, int capacity)
 
 // Block-wide sum of seq_tiles over sequences [0, n); every thread gets it.
 // Uses `red` (>= 32 int64) of shared scratch.  All threads must call it.
+// `groups` > 1: unit b of n is group b % groups of sequence b / groups (its
+// length is kv_len[b / groups]).
 __device__ __forceinline__ int64_t block_tile_sum(const int32_t *kv_len, int n, int q_len, int capacity,
-                                                  int64_t *red)
+                                                  int64_t *red, int groups = 1)
 {
     int64_t acc = 0;
-    for (int b = threadIdx.x; b < n; b += blockDim.x) acc += seq_tiles(kv_len[b], q_len, capacity);
+    for (int b = threadIdx.x; b < n; b += blockDim.x) acc += seq_tiles(kv_len[b / groups], q_len, capacity);
     for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     __syncthreads();
@@ -160,11 +162,11 @@ __device__ __forceinline__ int64_t block_tile_sum(const int32_t *kv_len, int n, 
 // One pass over the lengths: *total = all sequences' tiles, *before = the
 // tiles of sequences 0 .. b-1 (block-wide; every thread gets both).
 __device__ __forceinline__ void block_tile_sums(const int32_t *kv_len, int n, int b, int q_len, int capacity,
-                                                int64_t *red, int64_t *total, int64_t *before)
+                                                int64_t *red, int64_t *total, int64_t *before, int groups = 1)
 {
     int64_t acc = 0, pre = 0;
     for (int i = threadIdx.x; i < n; i += blockDim.x) {
-        const int64_t t = seq_tiles(kv_len[i], q_len, capacity);
+        const int64_t t = seq_tiles(kv_len[i / groups], q_len, capacity);
         acc += t;
         if (i < b) pre += t;
     }
@@ -198,14 +200,14 @@ __device__ __forceinline__ void block_tile_sums(const int32_t *kv_len, int n, in
 // result, read as a signed fraction x in [-1, 1), is the angle pi * x that
 // sincospif evaluates in fp32.  No fp64 arithmetic runs on the device.
 struct RopeTurns {
-    uint64_t f[32];  // d_rope / 2 <= 32 frequencies
+    uint64_t f[64];  // d / 2 <= 64 frequencies (positional keys of MLA, whole GQA heads up to 128)
 };
 
 inline RopeTurns rope_turns(int d_rope, float base)
 {
     RopeTurns t{};
     const double two_pi = 6.283185307179586476925286766559;
-    for (int k = 0; k < d_rope / 2 && k < 32; ++k) {
+    for (int k = 0; k < d_rope / 2 && k < 64; ++k) {
         const double theta = pow(static_cast<double>(base), -2.0 * k / d_rope);  // <= 1
         t.f[k] = static_cast<uint64_t>(ldexp(theta / two_pi, 64));                // < 2^62
     }

@@ -30,8 +30,12 @@ struct AttnArgs {
     unsigned *status;
 };
 
+// groups > 1: `batch` counts (sequence, KV group) units, entry rows [unit, n_new, .],
+// start_pos indexed by sequence (unit / groups); rank = value width, d_rope =
+// key width (the original-GQA cache).
 cudaError_t launch_append(const mla_dims &d, const CacheView &c, int batch, int n_new, const void *c_new,
-                          const void *kr_new, const int32_t *start_pos, unsigned *status, cudaStream_t st);
+                          const void *kr_new, const int32_t *start_pos, unsigned *status, cudaStream_t st,
+                          int groups = 1);
 
 cudaError_t launch_absorb(const mla_dims &d, int batch, int q_len, const void *q_nope, const void *q_pe,
                           const int32_t *kv_len, const void *w_uk, void *q_abs, unsigned *status,
@@ -50,9 +54,11 @@ struct TcShape {
 TcShape attn_tc_shape(int rows);
 cudaError_t launch_attn_tc(const AttnArgs &a, cudaStream_t st);
 
+// `groups` > 1: unit b of `batch` is KV group b % groups of sequence b / groups
+// (the original-GQA path); its length is kv_len[b / groups].
 cudaError_t launch_combine(int batch, int q_len, int num_heads, int rank, int max_kv, int num_splits,
                            const int32_t *kv_len, const float *o_part, const float *lse_part, float *o_lat,
-                           float *lse, cudaStream_t st);
+                           float *lse, cudaStream_t st, int groups = 1);
 
 cudaError_t launch_out_proj(const mla_dims &d, int batch, int q_len, const float *o_lat, const void *w_uv,
                             const void *w_o, void *o, void *out, unsigned *status, cudaStream_t st);
@@ -90,6 +96,21 @@ cudaError_t launch_project(const mla_dims &d, const CacheView &c, int batch, int
 cudaError_t launch_acceptance(int rows, int vocab, int dtype, const void *draft, const void *target, int64_t stride,
                               float *alpha, int32_t *argmax_d, int32_t *argmax_t, int32_t *greedy, unsigned *status,
                               cudaStream_t st);
+
+// Original-GQA decode attention (mla_gqa_decode_attn): per (sequence, KV
+// group) unit b * G + g, keys in cache.k_rope and values in cache.c_kv.
+struct GqaLaunch {
+    int batch, q_len, groups, hpg, head_dim, max_kv, num_splits;
+    float sm_scale;
+    int rope_style;
+    float rope_base;
+    const int32_t *kv_len;
+    const void *q;        // bf16 [B, q_len, H, head_dim], not rotated
+    float *o_part, *lse_part;
+    unsigned *status;
+    CacheView cache;
+};
+cudaError_t launch_gqa_attn(const GqaLaunch &g, cudaStream_t st);
 
 cudaError_t launch_selftest_wait(int64_t limit_ns, unsigned *status, cudaStream_t st);
 
