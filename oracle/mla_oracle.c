@@ -505,7 +505,7 @@ typedef struct {
 
 /* New keys and values of every (sequence, group) at positions start_pos[b] + k:
  * the key rotated in fp64 and rounded once to bf16, the value copied.
- *   k_new [batch, G, n_new, d_k], v_new [batch, G, n_new, d_v] bf16 */
+ *   k_new [batch, n_new, G, d_k], v_new [batch, n_new, G, d_v] bf16 */
 int orc_gqa_append(const orc_gqa_dims *d, const orc_cache *c, int batch, int n_new, const uint16_t *k_new,
                    const uint16_t *v_new, const int32_t *start_pos)
 {
@@ -517,7 +517,7 @@ int orc_gqa_append(const orc_gqa_dims *d, const orc_cache *c, int batch, int n_n
     for (int b = 0; b < batch && !err; ++b)
         for (int g = 0; g < G && !err; ++g)
             for (int k = 0; k < n_new && !err; ++k) {
-                const int64_t pos = (int64_t)start_pos[b] + k, e0 = ((int64_t)(b * G + g) * n_new + k);
+                const int64_t pos = (int64_t)start_pos[b] + k, e0 = ((int64_t)b * n_new + k) * G + g;
                 int64_t co, ro;
                 err = tok_offsets(c, b * G + g, pos, &co, &ro);
                 if (err) break;
@@ -583,4 +583,27 @@ int orc_gqa_decode(const orc_gqa_dims *d, const orc_cache *c, int batch, int q_l
         free(qr);
     }
     return err;
+}
+
+/* Forward value of the E2E functional-reconstruction loss of one layer
+ * (Sec. 4.1): the masked mean-squared error between the converted MLA
+ * block's post-W_O output and the frozen original block's,
+ *   L = sum_t M_t sum_d (A_MLA[t, d] - A_orig[t, d])^2 / (D sum_t M_t),
+ * over rows t (tokens) with mask M_t in {0, 1} (mask NULL: every row counts).
+ * A row set with no counted row gives 0.  a_mla, a_orig [rows, D] fp64. */
+int orc_e2e_loss(int rows, int hidden, const double *a_mla, const double *a_orig, const uint8_t *mask,
+                 double *loss)
+{
+    if (rows < 0 || hidden <= 0 || !loss) return ORC_BAD_ARG;
+    double num = 0.0, den = 0.0;
+    for (int t = 0; t < rows; ++t) {
+        if (mask && !mask[t]) continue;
+        for (int e = 0; e < hidden; ++e) {
+            const double d = a_mla[(int64_t)t * hidden + e] - a_orig[(int64_t)t * hidden + e];
+            num += d * d;
+        }
+        den += 1.0;
+    }
+    *loss = den > 0.0 ? num / ((double)hidden * den) : 0.0;
+    return ORC_OK;
 }

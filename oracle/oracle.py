@@ -154,6 +154,8 @@ def configure(lib):
     lib.orc_gqa_decode.restype = ctypes.c_int
     lib.orc_gqa_decode.argtypes = [ctypes.POINTER(_GqaDims), ctypes.POINTER(_Cache), ctypes.c_int, ctypes.c_int,
                                    vp, vp, vp, vp]
+    lib.orc_e2e_loss.restype = ctypes.c_int
+    lib.orc_e2e_loss.argtypes = [ctypes.c_int, ctypes.c_int, vp, vp, vp, vp]
     lib.orc_mla_decode.restype = ctypes.c_int
     lib.orc_mla_decode.argtypes = [ctypes.POINTER(_Dims), ctypes.POINTER(_Cache), ctypes.c_int,
                                    ctypes.c_int, vp, vp, vp, vp, vp, vp, vp, ctypes.c_int,
@@ -341,11 +343,11 @@ def acceptance(draft: np.ndarray, target: np.ndarray) -> dict:
 
 
 def gqa_append(dims: GqaDims, cache: Cache, k_new: np.ndarray, v_new: np.ndarray, start_pos) -> None:
-    """Original GQA cache append (Sec. 3.1): keys [B, G, n, d_k] rotated to
-    their positions (one bf16 rounding), values [B, G, n, d_v] copied; the
+    """Original GQA cache append (Sec. 3.1): keys [B, n, G, d_k] rotated to
+    their positions (one bf16 rounding), values [B, n, G, d_v] copied; the
     cache's c_kv holds values, k_rope keys, block (or table row) b * G + g."""
     k_new, v_new, start_pos = _u16(k_new), _u16(v_new), _i32(start_pos)
-    batch, n_new = k_new.shape[0], k_new.shape[2]
+    batch, n_new = k_new.shape[0], k_new.shape[1]
     _check(_load().orc_gqa_append(ctypes.byref(dims._c()), ctypes.byref(cache._c()), batch, n_new,
                                   k_new.ctypes.data, v_new.ctypes.data, start_pos.ctypes.data), "gqa_append")
 
@@ -360,3 +362,15 @@ def gqa_decode(dims: GqaDims, cache: Cache, q: np.ndarray, kv_len) -> dict:
     _check(_load().orc_gqa_decode(ctypes.byref(dims._c()), ctypes.byref(cache._c()), batch, q_len, kv_len.ctypes.data,
                                   q.ctypes.data, o.ctypes.data, lse.ctypes.data), "gqa_decode")
     return {"o": o, "lse": lse}
+
+
+def e2e_loss(a_mla: np.ndarray, a_orig: np.ndarray, mask: Optional[np.ndarray] = None) -> float:
+    """E2E functional-reconstruction loss forward (Sec. 4.1): masked MSE of the
+    two blocks' post-W_O outputs [rows, D] (fp64), mask [rows] in {0, 1}."""
+    a = np.ascontiguousarray(a_mla, dtype=np.float64).reshape(-1, a_mla.shape[-1])
+    b = np.ascontiguousarray(a_orig, dtype=np.float64).reshape(-1, a_orig.shape[-1])
+    m = None if mask is None else np.ascontiguousarray(mask, dtype=np.uint8).reshape(-1)
+    out = np.zeros(1)
+    _check(_load().orc_e2e_loss(a.shape[0], a.shape[1], a.ctypes.data, b.ctypes.data, _ptr(m), out.ctypes.data),
+           "e2e_loss")
+    return float(out[0])

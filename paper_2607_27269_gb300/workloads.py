@@ -35,7 +35,7 @@ cache per KV group) keeps the MLA workload's lengths, positions and page
 counts and draws from a fourth generator seeded with ``seed + 15485863``: the
 page permutation (paged), key and value caches ~ N(0, 1) (keys taken as
 already rotated), queries q [B, q_len, H, d] and this step's new keys and
-values [B, G, q_len, d] ~ N(0, 1).
+values [B, q_len, G, d] ~ N(0, 1).
 
 Inputs of the projection that precedes the step (``projection``) come from a
 second generator seeded with ``seed + 7919``, drawn in this order: hidden
@@ -275,8 +275,8 @@ class GqaWorkload:
     block_table: Optional[torch.Tensor]  # int32 [B * G, pages] (paged) or None
     num_pages: int
     q: torch.Tensor               # bf16 [B, q_len, H, d]
-    k_new: torch.Tensor           # bf16 [B, G, q_len, d] (not rotated)
-    v_new: torch.Tensor           # bf16 [B, G, q_len, d]
+    k_new: torch.Tensor           # bf16 [B, q_len, G, d] (not rotated)
+    v_new: torch.Tensor           # bf16 [B, q_len, G, d]
 
     @property
     def sm_scale(self) -> float:
@@ -314,7 +314,7 @@ def gqa(w: Workload, seed: int = 0) -> GqaWorkload:
     k_cache = _randn(gen, (blocks, block_tokens, d))
     v_cache = _randn(gen, (blocks, block_tokens, d))
     qq = _randn(gen, (B, q, H, d))
-    k_new = _randn(gen, (B, G, q, d))
-    v_new = _randn(gen, (B, G, q, d))
+    k_new = _randn(gen, (B, q, G, d))
+    v_new = _randn(gen, (B, q, G, d))
     return GqaWorkload(s, H, G, d, w.kv_len.clone(), w.start_pos.clone(), cap, k_cache, v_cache, bt, num_pages, qq,
                        k_new, v_new)

@@ -44,6 +44,9 @@ MUTANTS = {
                           "const int g = h % G;\n        const int64_t p = (int64_t)kv_len[b] - q_len + i;"),
     "gqa_value_block": ("tok_offsets(c, b * G + g, j, &co, &ro);\n                acc += exp",
                         "tok_offsets(c, b * G + (g + 1) % G, j, &co, &ro);\n                acc += exp"),
+    "e2e_loss_counts_masked_rows": ("if (mask && !mask[t]) continue;", "if (mask && mask[t] > 1) continue;"),
+    "e2e_loss_missing_hidden": ("*loss = den > 0.0 ? num / ((double)hidden * den) : 0.0;",
+                                "*loss = den > 0.0 ? num / den : 0.0;"),
     "output_projection_index": ("acc += orc_bf16_value(w[h * dv + e]) * o[(row0 + h) * dv + e];",
                                 "acc += orc_bf16_value(w[e * H + h]) * o[(row0 + h) * dv + e];"),
 }

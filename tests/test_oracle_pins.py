@@ -614,7 +614,7 @@ def test_gqa_oracle_matches_sdpa(paged):
         for t in range(int(gw.start_pos[b]), kv):          # appended keys: one rounding of the exact rotation
             for g in range(G):
                 k, _ = _gqa_logical(gw, cache, b, g, t)
-                exact = rope_complex(bf16_to_f64(bits(gw.k_new))[b, g, t - int(gw.start_pos[b])], t)
+                exact = rope_complex(bf16_to_f64(bits(gw.k_new))[b, t - int(gw.start_pos[b]), g], t)
                 ulp = 2.0 ** (np.floor(np.log2(np.maximum(np.abs(exact), 1e-30))) - 7)
                 assert np.all(np.abs(k - exact) <= ulp / 2 + 1e-15)
         K = np.stack([np.stack([_gqa_logical(gw, cache, b, g, t)[0] for t in range(kv)]) for g in range(G)])
@@ -630,3 +630,25 @@ def test_gqa_oracle_matches_sdpa(paged):
         logits = np.einsum("qhd,htd->hqt", Q, np.repeat(K, H // G, axis=0)) * gw.sm_scale
         logits = np.where(mask[None], logits, -np.inf)
         np.testing.assert_allclose(res["lse"][b].T, scipy.special.logsumexp(logits, axis=2), rtol=1e-12, atol=1e-12)
+
+
+# ---------------------------------------------------------------- E2E loss forward (Sec. 4.1)
+
+def test_e2e_loss_closed_forms_and_invariances():
+    g = np.random.default_rng(7)
+    a = g.standard_normal((9, 40))
+    b = g.standard_normal((9, 40))
+    mask = (g.random(9) < 0.6).astype(np.uint8)
+    mask[0] = 1
+    assert orc.e2e_loss(a, a, mask) == 0.0                                     # identical blocks
+    np.testing.assert_allclose(orc.e2e_loss(a + 0.3, a, mask), 0.09, rtol=1e-13)  # constant offset c: c^2
+    base = orc.e2e_loss(a, b, mask)
+    np.testing.assert_allclose(orc.e2e_loss(2.5 * a, 2.5 * b, mask), 6.25 * base, rtol=1e-13)  # scaling
+    b2 = b.copy()
+    b2[mask == 0] += 100.0                                                     # masked-out rows do not count
+    assert orc.e2e_loss(a, b2, mask) == base
+    one = np.zeros(9, dtype=np.uint8)
+    one[3] = 1                                                                 # one row: its mean square
+    np.testing.assert_allclose(orc.e2e_loss(a, b, one), np.mean((a[3] - b[3]) ** 2), rtol=1e-13)
+    np.testing.assert_allclose(orc.e2e_loss(a, b), np.mean((a - b) ** 2), rtol=1e-13)  # no mask: every row
+    assert orc.e2e_loss(a, b, np.zeros(9, dtype=np.uint8)) == 0.0             # no counted row
