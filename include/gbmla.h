@@ -242,7 +242,7 @@ typedef struct mla_gqa_dims {
 
 /* New keys and values of every (sequence, group) at positions start_pos[b] + k:
  * keys rotated in fp32 and rounded once to bf16, values copied.
- *   k_new, v_new [batch, G, n_new, head_dim] bf16; start_pos [batch] int32.
+ *   k_new, v_new [batch, n_new, G, head_dim] bf16; start_pos [batch] int32.
  * Faults as for mla_cache_append. */
 mla_status mla_gqa_append(const mla_gqa_dims *dims, const mla_cache *cache, int32_t batch, int32_t n_new,
                           const void *k_new, const void *v_new, const int32_t *start_pos, void *stream);
@@ -258,12 +258,41 @@ mla_status mla_gqa_workspace_size(const mla_gqa_dims *dims, int32_t batch, int32
  * of group g = h / (H/G),
  *   o = sum_j softmax_j(sm_scale (R_p q[b,i,h]) . K[b,g,j]) V[b,g,j],  j <= p
  * q [batch, q_len, H, head_dim] bf16 (not rotated), q_len * H/G <= 128;
- * o_part / lse_part sized by mla_gqa_workspace_size; outputs in group-major
- * order: o [batch, G, q_len, H/G, head_dim] fp32, lse [batch, G, q_len, H/G]
- * fp32 (natural log) or NULL. */
+ * o_part / lse_part sized by mla_gqa_workspace_size; outputs
+ * o [batch, q_len, H, head_dim] fp32, lse [batch, q_len, H] fp32 (natural
+ * log) or NULL. */
 mla_status mla_gqa_decode_attn(const mla_gqa_dims *dims, const mla_cache *cache, int32_t batch, int32_t q_len,
                                const int32_t *kv_len, int32_t max_kv_len, const void *q, int32_t num_splits,
                                float *o_part, float *lse_part, float *o, float *lse, void *stream);
+
+/* Projections of the original GQA layer (Sec. 3.1, Eq. 1), bf16 results:
+ *   q [batch, n_new, H, head_dim]         = h W_Q^T   (W_Q [H head_dim, hidden])
+ *   k_new, v_new [batch, n_new, G, head_dim] = h W_K^T, h W_V^T (W_K, W_V [G head_dim, hidden])
+ * h [batch, n_new, hidden] bf16, hidden a multiple of 8; every pointer 16-byte
+ * aligned.  (q is not rotated; mla_gqa_append rotates the keys, the attention
+ * the queries.) */
+mla_status mla_gqa_project(const mla_gqa_dims *dims, int32_t batch, int32_t n_new, int32_t hidden, const void *h,
+                           const void *w_q, const void *w_k, const void *w_v, void *q, void *k_new, void *v_new,
+                           void *stream);
+
+/* Output projection of the original GQA layer: out [batch, q_len, hidden] =
+ * W_O concat_h o (concat index h head_dim + e), o [batch, q_len, H, head_dim]
+ * fp32 (as mla_gqa_decode_attn writes it), W_O [hidden, H head_dim] bf16; the
+ * same frozen W_O serves the converted MLA layer (Sec. 4.1). */
+mla_status mla_gqa_out_proj(const mla_gqa_dims *dims, int32_t batch, int32_t q_len, int32_t hidden, const float *o,
+                            const void *w_o, void *out, void *stream);
+
+/* Forward value of the E2E functional-reconstruction loss of one layer
+ * (Sec. 4.1): the masked mean-squared error between the converted MLA
+ * block's post-W_O output and the frozen original block's,
+ *   loss = sum_t M_t sum_d (a_mla[t, d] - a_orig[t, d])^2 / (hidden sum_t M_t)
+ * a_mla, a_orig [rows, hidden] bf16 (hidden a multiple of 8, 16-byte
+ * aligned); mask [rows] uint8 (nonzero = counted) or NULL (every row); loss:
+ * one device float (0 when no row counts).  fp32 products, fp64 sums, added
+ * in a fixed order: the same bits on every run.  Backward and training are
+ * not part of this library. */
+mla_status mla_e2e_loss(int32_t rows, int32_t hidden, const void *a_mla, const void *a_orig, const uint8_t *mask,
+                        float *loss, void *stream);
 
 /* mla_decode_attn followed by mla_combine, for callers that cannot allocate
  * device memory: code that runs where an allocation is not allowed (inside a

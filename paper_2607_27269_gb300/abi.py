@@ -20,7 +20,8 @@ from . import build as _build
 MLA_OK, MLA_ERR_INVALID_ARG, MLA_ERR_UNSUPPORTED, MLA_ERR_CUDA, MLA_ERR_DEVICE_BOUNDS, MLA_ERR_DEVICE_TIMEOUT = range(6)
 SPLIT_TILE = 128
 EXPORTS = ("mla_workspace_size", "mla_cache_append", "mla_project_append", "mla_acceptance_stats",
-           "mla_gqa_append", "mla_gqa_workspace_size", "mla_gqa_decode_attn", "mla_absorb_q", "mla_decode_attn", "mla_combine",
+           "mla_gqa_append", "mla_gqa_workspace_size", "mla_gqa_decode_attn", "mla_gqa_project", "mla_gqa_out_proj",
+           "mla_e2e_loss", "mla_absorb_q", "mla_decode_attn", "mla_combine",
            "mla_out_proj", "mla_check_status", "mla_selftest_wait_timeout", "mla_decode_attn_noalloc",
            "mla_status_str", "mla_last_error")
 
@@ -79,6 +80,9 @@ def lib(auto_build: bool = True):
             L.mla_absorb_q.argtypes = [P(MlaDims), i32, i32, vp, vp, vp, vp, vp, vp]
             L.mla_acceptance_stats.argtypes = [i32, i32, i32, vp, vp, i64, vp, vp, vp, vp, vp]
             L.mla_gqa_append.argtypes = [P(MlaGqaDims), P(MlaCache), i32, i32, vp, vp, vp, vp]
+            L.mla_gqa_project.argtypes = [P(MlaGqaDims), i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp]
+            L.mla_gqa_out_proj.argtypes = [P(MlaGqaDims), i32, i32, i32, vp, vp, vp, vp]
+            L.mla_e2e_loss.argtypes = [i32, i32, vp, vp, vp, vp, vp]
             L.mla_gqa_workspace_size.argtypes = [P(MlaGqaDims), i32, i32, i32, i32, P(sz), P(sz), P(i32)]
             L.mla_gqa_decode_attn.argtypes = [P(MlaGqaDims), P(MlaCache), i32, i32, vp, i32, vp, i32, vp, vp, vp, vp,
                                               vp]
@@ -208,8 +212,8 @@ class GqaDims:
 
 def gqa_append(dims: GqaDims, cache: Cache, k_new: torch.Tensor, v_new: torch.Tensor, start_pos: torch.Tensor,
                stream=None):
-    """k_new / v_new [B, G, n, head_dim] into the GQA cache (keys in cache.k_rope, values in cache.c_kv)."""
-    batch, n_new = k_new.shape[0], k_new.shape[2]
+    """k_new / v_new [B, n, G, head_dim] into the GQA cache (keys in cache.k_rope, values in cache.c_kv)."""
+    batch, n_new = k_new.shape[0], k_new.shape[1]
     _check("mla_gqa_append", lib().mla_gqa_append(ctypes.byref(dims.c()), ctypes.byref(cache.c()), batch, n_new,
                                                   _p(k_new), _p(v_new), _p(start_pos), _stream(stream)))
 
@@ -224,7 +228,7 @@ def gqa_workspace_size(dims: GqaDims, batch: int, q_len: int, max_kv_len: int, n
 
 class GqaStep:
     """GQA decode attention with its partial buffers allocated once:
-    o [B, G, q_len, H/G, head_dim] fp32 (group-major), lse [B, G, q_len, H/G]."""
+    o [B, q_len, H, head_dim] fp32, lse [B, q_len, H]."""
 
     def __init__(self, dims: GqaDims, cache: Cache, batch: int, q_len: int, max_kv_len: int, num_splits: int = 0):
         self.dims, self.cache, self.batch, self.q_len, self.max_kv_len = dims, cache, batch, q_len, max_kv_len
@@ -233,8 +237,8 @@ class GqaStep:
         G, hpg, d = dims.num_kv_groups, dims.num_heads // dims.num_kv_groups, dims.head_dim
         self.o_part = torch.empty(max(ob // 4, 1), dtype=torch.float32, device=dev)
         self.lse_part = torch.empty(max(lb // 4, 1), dtype=torch.float32, device=dev)
-        self.o = torch.empty(batch, G, q_len, hpg, d, dtype=torch.float32, device=dev)
-        self.lse = torch.empty(batch, G, q_len, hpg, dtype=torch.float32, device=dev)
+        self.o = torch.empty(batch, q_len, dims.num_heads, d, dtype=torch.float32, device=dev)
+        self.lse = torch.empty(batch, q_len, dims.num_heads, dtype=torch.float32, device=dev)
 
     def __call__(self, q: torch.Tensor, kv_len: torch.Tensor, stream=None):
         _check("mla_gqa_decode_attn", lib().mla_gqa_decode_attn(
@@ -242,6 +246,64 @@ class GqaStep:
             self.max_kv_len, _p(q), self.num_splits, _p(self.o_part), _p(self.lse_part), _p(self.o), _p(self.lse),
             _stream(stream)))
         return self.o
+
+
+def gqa_project(dims: GqaDims, h: torch.Tensor, w_q, w_k, w_v, q, k_new, v_new, stream=None):
+    """q [B, n, H, d], k_new / v_new [B, n, G, d] = h [B, n, D] times W_Q^T, W_K^T, W_V^T (bf16)."""
+    batch, n_new, hidden = h.shape
+    _check("mla_gqa_project", lib().mla_gqa_project(ctypes.byref(dims.c()), batch, n_new, hidden, _p(h), _p(w_q),
+                                                    _p(w_k), _p(w_v), _p(q), _p(k_new), _p(v_new), _stream(stream)))
+
+
+def gqa_out_proj(dims: GqaDims, o: torch.Tensor, w_o: torch.Tensor, out: torch.Tensor, stream=None):
+    """out [B, q, D] = W_O concat_h o (o fp32 [B, q, H, d])."""
+    batch, q_len = o.shape[:2]
+    _check("mla_gqa_out_proj", lib().mla_gqa_out_proj(ctypes.byref(dims.c()), batch, q_len, w_o.shape[0], _p(o),
+                                                      _p(w_o), _p(out), _stream(stream)))
+
+
+def e2e_loss(a_mla: torch.Tensor, a_orig: torch.Tensor, mask: Optional[torch.Tensor] = None,
+             loss: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """E2E functional-reconstruction loss forward (masked MSE of the two blocks'
+    post-W_O outputs, bf16 [.., D]); returns a one-element fp32 device tensor."""
+    hidden = a_mla.shape[-1]
+    rows = a_mla.numel() // hidden
+    loss = torch.empty(1, dtype=torch.float32, device=a_mla.device) if loss is None else loss
+    _check("mla_e2e_loss", lib().mla_e2e_loss(rows, hidden, _p(a_mla), _p(a_orig), _p(mask), _p(loss),
+                                              _stream(stream)))
+    return loss
+
+
+class E2EForward:
+    """Forward of the E2E functional-reconstruction loss (Sec. 4.1) on one
+    chunk of calibration hidden states: the converted MLA layer (projection
+    into its latent cache, absorbed attention, W_UV, W_O) and the original GQA
+    layer (its projections, cache append, attention, the same frozen W_O) run
+    on the same h, and their post-W_O outputs meet in the masked MSE.  Every
+    buffer is allocated once here."""
+
+    def __init__(self, mla_step: "DecodeStep", gqa_dims: GqaDims, gqa_cache: Cache, hidden: int):
+        self.mla = mla_step
+        b, q = mla_step.batch, mla_step.q_len
+        dev = mla_step.q_abs.device
+        self.gqa_dims = gqa_dims
+        self.gqa = GqaStep(gqa_dims, gqa_cache, b, q, mla_step.max_kv_len)
+        d, H, G = gqa_dims.head_dim, gqa_dims.num_heads, gqa_dims.num_kv_groups
+        self.q = torch.empty(b, q, H, d, dtype=torch.bfloat16, device=dev)
+        self.k_new = torch.empty(b, q, G, d, dtype=torch.bfloat16, device=dev)
+        self.v_new = torch.empty(b, q, G, d, dtype=torch.bfloat16, device=dev)
+        self.out_orig = torch.empty(b, q, hidden, dtype=torch.bfloat16, device=dev)
+        self.loss = torch.empty(1, dtype=torch.float32, device=dev)
+
+    def __call__(self, h, mla_w, gqa_w, w_o, start_pos, kv_len, mask=None, stream=None):
+        """mla_w = (w_dkv, w_kr, w_q, w_uk, w_uv), gqa_w = (w_q, w_k, w_v); returns the loss tensor."""
+        w_dkv, w_kr, w_qm, w_uk, w_uv = mla_w
+        out_mla = self.mla.from_hidden(h, w_dkv, w_kr, w_qm, start_pos, kv_len, w_uk, w_uv, w_o, stream=stream)
+        gqa_project(self.gqa_dims, h, *gqa_w, self.q, self.k_new, self.v_new, stream)
+        gqa_append(self.gqa_dims, self.gqa.cache, self.k_new, self.v_new, start_pos, stream)
+        o = self.gqa(self.q, kv_len, stream)
+        gqa_out_proj(self.gqa_dims, o, w_o, self.out_orig, stream)
+        return e2e_loss(out_mla, self.out_orig, mask, self.loss, stream)
 
 
 def acceptance_stats(draft: torch.Tensor, target: torch.Tensor, alpha: Optional[torch.Tensor] = None,

@@ -20,7 +20,7 @@ BUILD_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libgbmla.so")
 LIB_TRACE = os.path.join(PKG, "libgbmla_trace.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["accept.cu", "api.cu", "append.cu", "absorb.cu", "attn_simt.cu", "attn_tc.cu", "combine.cu", "gemm.cu", "gqa.cu", "out_proj.cu"]
+SOURCES = ["accept.cu", "api.cu", "append.cu", "absorb.cu", "e2e.cu", "attn_simt.cu", "attn_tc.cu", "combine.cu", "gemm.cu", "gqa.cu", "out_proj.cu"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
               "-Xptxas", "-warn-spills"] + ARCH
 

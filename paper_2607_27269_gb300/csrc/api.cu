@@ -376,6 +376,85 @@ mla_status mla_gqa_decode_attn(const mla_gqa_dims *dims, const mla_cache *cache,
                                     o_part, lse_part, o, lse, st, g.groups));
 }
 
+mla_status mla_gqa_project(const mla_gqa_dims *dims, int32_t batch, int32_t n_new, int32_t hidden, const void *h,
+                           const void *w_q, const void *w_k, const void *w_v, void *q, void *k_new, void *v_new,
+                           void *stream)
+{
+    mla_dims d;
+    mla_status s = gqa_as_mla(dims, &d);
+    if (s != MLA_OK) return s;
+    if (batch < 0 || n_new < 0 || hidden <= 0 || hidden % 8) return MLA_ERR_INVALID_ARG;
+    if (batch == 0 || n_new == 0) return MLA_OK;
+    const void *ptrs[7] = {h, w_q, w_k, w_v, q, k_new, v_new};
+    for (const void *p : ptrs)
+        if (!p || !aligned16(p)) return MLA_ERR_INVALID_ARG;
+    if (static_cast<int64_t>(batch) * n_new > (1 << 24)) return MLA_ERR_UNSUPPORTED;
+    unsigned *status = nullptr;
+    if ((s = device_info(&status, nullptr)) != MLA_OK) return s;
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int M = batch * n_new, hd = dims->head_dim;
+    const int cols[3] = {dims->num_heads * hd, dims->num_kv_groups * hd, dims->num_kv_groups * hd};
+    const void *w[3] = {w_q, w_k, w_v};
+    void *outs[3] = {q, k_new, v_new};
+    for (int k = 0; k < 3; ++k) {
+        GroupGemm p;
+        p.M = M;
+        p.N = cols[k];
+        p.K = hidden;
+        p.G = 1;
+        p.hpg = 1;
+        p.blk = 1;
+        p.A = h;
+        p.a_f32 = 0;
+        p.lda = hidden;
+        p.B = w[k];
+        p.b_nmajor = 0;
+        p.C = outs[k];
+        p.ldc = cols[k];
+        p.status = status;
+        const cudaError_t e = launch_group_gemm(p, st);
+        if (e != cudaSuccess) return from_cuda(e);
+    }
+    return MLA_OK;
+}
+
+mla_status mla_gqa_out_proj(const mla_gqa_dims *dims, int32_t batch, int32_t q_len, int32_t hidden, const float *o,
+                            const void *w_o, void *out, void *stream)
+{
+    mla_dims d;
+    mla_status s = gqa_as_mla(dims, &d);
+    if (s != MLA_OK) return s;
+    if (batch < 0 || q_len < 0 || hidden <= 0 || hidden % 8) return MLA_ERR_INVALID_ARG;
+    if (batch == 0 || q_len == 0) return MLA_OK;
+    if (!o || !w_o || !out || !aligned16(o) || !aligned16(w_o) || !aligned16(out)) return MLA_ERR_INVALID_ARG;
+    unsigned *status = nullptr;
+    if ((s = device_info(&status, nullptr)) != MLA_OK) return s;
+    GroupGemm p;
+    p.M = batch * q_len;
+    p.N = hidden;
+    p.K = dims->num_heads * dims->head_dim;
+    p.G = 1;
+    p.hpg = 1;
+    p.blk = 1;
+    p.A = o;
+    p.a_f32 = 1;
+    p.lda = p.K;
+    p.B = w_o;
+    p.b_nmajor = 0;
+    p.C = out;
+    p.ldc = hidden;
+    p.status = status;
+    return from_cuda(launch_group_gemm(p, static_cast<cudaStream_t>(stream)));
+}
+
+mla_status mla_e2e_loss(int32_t rows, int32_t hidden, const void *a_mla, const void *a_orig, const uint8_t *mask,
+                        float *loss, void *stream)
+{
+    if (rows < 0 || hidden <= 0 || hidden % 8 || !loss) return MLA_ERR_INVALID_ARG;
+    if (rows > 0 && (!a_mla || !a_orig || !aligned16(a_mla) || !aligned16(a_orig))) return MLA_ERR_INVALID_ARG;
+    return from_cuda(launch_e2e_loss(rows, hidden, a_mla, a_orig, mask, loss, static_cast<cudaStream_t>(stream)));
+}
+
 mla_status mla_absorb_q(const mla_dims *dims, int32_t batch, int32_t q_len, const void *q_nope, const void *q_pe,
                         const int32_t *kv_len, const void *w_uk, void *q_abs, void *stream)
 {

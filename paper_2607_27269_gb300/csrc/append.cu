@@ -40,7 +40,8 @@ __global__ void __launch_bounds__(128) cache_append_kernel(CacheView c, int rank
     }
     uint16_t *crow = (uint16_t *)c.c_kv + blk * c.c_blk + slot * c.c_tok;
     uint16_t *rrow = (uint16_t *)c.k_rope + blk * c.r_blk + slot * c.r_tok;
-    const int64_t entry = static_cast<int64_t>(b) * n_new + k;
+    const int64_t entry = groups == 1 ? static_cast<int64_t>(b) * n_new + k
+                                      : (static_cast<int64_t>(b / groups) * n_new + k) * groups + b % groups;
     const uint4 *src = reinterpret_cast<const uint4 *>(c_new + entry * rank);
     for (int v = threadIdx.x; v < rank / 8; v += blockDim.x) reinterpret_cast<uint4 *>(crow)[v] = src[v];
 

@@ -99,10 +99,14 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(int batch, int
         const int row = row0 + r * rpb;
         if (row >= rows) continue;
         const float inv = wsum[r] > 0.f ? 1.f / wsum[r] : 0.f;
-        reinterpret_cast<float4 *>(o_lat + (static_cast<int64_t>(b) * rows + row) * rank)[part] =
+        // output row: (b, row) for the MLA path; for groups > 1, row = i * H + head of
+        // sequence b / groups, head = (b % groups) * H + h (rows of a unit are (i, h))
+        const int64_t orow = groups == 1 ? static_cast<int64_t>(b) * rows + row
+                                         : (static_cast<int64_t>(b / groups) * q_len + row / H) * (groups * H) +
+                                               (b % groups) * H + row % H;
+        reinterpret_cast<float4 *>(o_lat + orow * rank)[part] =
             make_float4(acc[r].x * inv, acc[r].y * inv, acc[r].z * inv, acc[r].w * inv);
-        if (lse_out && part == 0)
-            lse_out[static_cast<int64_t>(b) * rows + row] = wsum[r] > 0.f ? m[r] + logf(wsum[r]) : -INFINITY;
+        if (lse_out && part == 0) lse_out[orow] = wsum[r] > 0.f ? m[r] + logf(wsum[r]) : -INFINITY;
     }
 }
 

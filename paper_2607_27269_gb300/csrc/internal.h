@@ -30,7 +30,8 @@ struct AttnArgs {
     unsigned *status;
 };
 
-// groups > 1: `batch` counts (sequence, KV group) units, entry rows [unit, n_new, .],
+// groups > 1: `batch` counts (sequence, KV group) units, entry rows
+// [sequence, n_new, group, .] (token-major, as a projection writes them),
 // start_pos indexed by sequence (unit / groups); rank = value width, d_rope =
 // key width (the original-GQA cache).
 cudaError_t launch_append(const mla_dims &d, const CacheView &c, int batch, int n_new, const void *c_new,
@@ -55,7 +56,9 @@ TcShape attn_tc_shape(int rows);
 cudaError_t launch_attn_tc(const AttnArgs &a, cudaStream_t st);
 
 // `groups` > 1: unit b of `batch` is KV group b % groups of sequence b / groups
-// (the original-GQA path); its length is kv_len[b / groups].
+// (the original-GQA path; num_heads = heads per group); its length is
+// kv_len[b / groups], and its rows (i, h) go to head (b % groups) * num_heads + h
+// of row (sequence, i) of o_lat / lse, i.e. [B, q_len, G * num_heads, rank].
 cudaError_t launch_combine(int batch, int q_len, int num_heads, int rank, int max_kv, int num_splits,
                            const int32_t *kv_len, const float *o_part, const float *lse_part, float *o_lat,
                            float *lse, cudaStream_t st, int groups = 1);
@@ -111,6 +114,10 @@ struct GqaLaunch {
     CacheView cache;
 };
 cudaError_t launch_gqa_attn(const GqaLaunch &g, cudaStream_t st);
+
+// E2E loss forward (mla_e2e_loss): a_mla, a_orig bf16 [rows, hidden], mask [rows] or null.
+cudaError_t launch_e2e_loss(int rows, int hidden, const void *a_mla, const void *a_orig, const uint8_t *mask,
+                            float *loss, cudaStream_t st);
 
 cudaError_t launch_selftest_wait(int64_t limit_ns, unsigned *status, cudaStream_t st);
 

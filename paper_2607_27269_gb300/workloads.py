@@ -318,3 +318,24 @@ def gqa(w: Workload, seed: int = 0) -> GqaWorkload:
     v_new = _randn(gen, (B, q, G, d))
     return GqaWorkload(s, H, G, d, w.kv_len.clone(), w.start_pos.clone(), cap, k_cache, v_cache, bt, num_pages, qq,
                        k_new, v_new)
+
+
+@dataclass
+class GqaProjection:
+    """Projection weights of the original GQA layer (its W_O is the shared one)."""
+    w_q: torch.Tensor             # bf16 [H d, D]
+    w_k: torch.Tensor             # bf16 [G d, D]
+    w_v: torch.Tensor             # bf16 [G d, D]
+
+
+def gqa_projection(w: Workload, seed: int = 0, hidden: Optional[int] = None) -> GqaProjection:
+    """W_Q, W_K, W_V ~ N(0, 1/sqrt(D)) of the original layer at ``w``'s shape
+    (a fifth generator, seed + 32452843); D as in ``projection``."""
+    s = w.shape
+    D = hidden if hidden is not None else (s.hidden if s.hidden > 0 else 256)
+    gen = torch.Generator(device="cpu")
+    gen.manual_seed(seed + 32452843)
+    std = 1.0 / math.sqrt(D)
+    d = s.d_v
+    return GqaProjection(_randn(gen, (s.num_heads * d, D), std), _randn(gen, (s.num_kv_groups * d, D), std),
+                         _randn(gen, (s.num_kv_groups * d, D), std))
