@@ -257,6 +257,7 @@ def run_ours(args, rank, world, local):
         proj = measure_projection(args, w, dws, stream, dev, l2, peaks=load_peaks())
         accept = measure_acceptance(args, stream, dev, l2, peaks=load_peaks())
         gqa = measure_gqa(args, w, dws, steps, stream, dev, l2, peaks=load_peaks())
+        e2e_fwd = measure_e2e_forward(args, w, stream, dev)
 
         # ---- end to end through the public API with host buffers: the step's
         # inputs (queries, new entries, lengths, positions) packed in one pinned
@@ -348,8 +349,43 @@ def run_ours(args, rank, world, local):
         "project_append": proj,
         "acceptance_stats": accept,
         "gqa_comparison": gqa,
+        "e2e_loss_forward": e2e_fwd,
     }
     return line, w
+
+
+def measure_e2e_forward(args, w, stream, dev):
+    """One forward of the E2E functional-reconstruction loss (Sec. 4.1) on the
+    workload's new tokens: the converted MLA layer from hidden states and the
+    original GQA layer on the same states, the shared W_O, the masked MSE.
+    Timed as a CUDA graph of back-to-back forwards on one copy (the caches stay
+    resident; the new entries are rewritten in place each time)."""
+    import torch
+    from paper_2607_27269_gb300 import abi
+    from paper_2607_27269_gb300 import workloads as wl
+
+    s = w.shape
+    p = wl.projection(w, seed=args.seed)
+    gw = wl.gqa(w, seed=args.seed)
+    gp = wl.gqa_projection(w, seed=args.seed)
+    if w.w_o is None:
+        return {"skipped": "no output projection at this shape"}
+    dw = abi.to_device(w, dev)
+    step = abi.DecodeStep(dw.dims, dw.cache, dw.batch, dw.q_len, dw.max_kv_len)
+    gdims = abi.GqaDims(gw.num_heads, gw.num_kv_groups, gw.d, gw.sm_scale, s.rope_style, s.rope_base)
+    bt = None if gw.block_table is None else gw.block_table.to(dev)
+    gcache = abi.Cache(gw.v_cache.to(dev), gw.k_cache.to(dev), gw.capacity, bt, s.page_size if s.paged else 0,
+                       gw.num_pages)
+    fwd = abi.E2EForward(step, gdims, gcache, p.hidden)
+    mla_w = tuple(t.to(dev) for t in (p.w_dkv, p.w_kr, p.w_q, w.w_uk, w.w_uv))
+    gqa_w = tuple(t.to(dev) for t in (gp.w_q, gp.w_k, gp.w_v))
+    h, w_o = p.h.to(dev), w.w_o.to(dev)
+    us = _graph_time_us(lambda i: fwd(h, mla_w, gqa_w, w_o, dw.start_pos, dw.kv_len, stream=stream), 16, stream, dev)
+    code = abi.check_status(stream)
+    if code != abi.MLA_OK:
+        raise RuntimeError(f"device status after the E2E forward: {abi.status_name(code)}")
+    return {"us_per_forward": round(us, 3), "tokens": int(w.kv_len.numel() * s.q_len), "hidden": p.hidden,
+            "loss": round(float(fwd.loss.item()), 6)}
 
 
 def _graph_time_us(launch, n_launch, stream, dev):
