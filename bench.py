@@ -307,7 +307,7 @@ def run_ours(args, rank, world, local):
     attn_avg_ms = sum(attn_ms) / len(attn_ms)
     peaks = load_peaks()
     achieved = cache_bytes / (attn_avg_ms * 1e-3) / 1e9
-    launches_per_step = 1 + 2 + 1 + 1 + (2 if shape.hidden else 1)
+    launches_per_step = 1 + 1 + 1 + 1 + (2 if shape.hidden else 1)  # append, absorb, attention, combine, W_UV (+ W_O)
     line = {
         "metric": METRIC,
         "value": round(total_bytes / (max_ms * 1e-3) / 1e9, 2),

@@ -36,6 +36,10 @@ __device__ __forceinline__ int64_t phys_row(const GroupGemm &p, int g, int m)
 
 // Epilogue arguments of the projection (PROJ): column tiles [0, tiles_lat)
 // hold the latent, tile tiles_lat the positional key, the rest the queries.
+// The absorption GEMM (not PROJ) reuses it for the positional query: when
+// rope_src is set, the CTAs of each row tile also write
+// C[row, rank .. rank + d_rope) = R_p q_pe[row] for the rows of that tile,
+// p = kv_len[b] - q_len + i for row (b, i, head) (rows in [B, q_len, heads] order).
 struct ProjEpi {
     CacheView cache;
     const int32_t *start_pos;
@@ -44,6 +48,9 @@ struct ProjEpi {
     RopeTurns turns;
     int tiles_lat;
     uint32_t box_bytes[3];  // weight-tile bytes of the three column regions
+    const uint16_t *rope_src;  // absorption: q_pe [B, q_len, heads, d_rope], or null
+    const int32_t *kv_len;
+    int q_len;
 };
 
 __device__ __forceinline__ void store16_bf16(uint16_t *dst, const uint32_t (&v)[16])
@@ -367,6 +374,46 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
                 if (lane == 0) tc::mbar_arrive(smem_u32(&bars.conv_done[s]));
             }
         }
+        if (!PROJ && pe.rope_src) {
+            // ---- the absorption's positional query, while the MMAs run.  The
+            // tile's rows are whole (b, i) blocks of hpg heads (row m of group g
+            // is head g hpg + m % hpg of token m / hpg), which share one
+            // position: an item is one (token, pair) with one angle, applied to
+            // the pair of every head of the group.  The items of this row tile
+            // are spread over the CTAs that share it (column tiles, K shares).
+            const int half = pe.d_rope / 2, hpg = p.hpg;
+            const int slots = static_cast<int>(gridDim.y) * ks, slot = static_cast<int>(blockIdx.y) * ks + kz;
+            const int tok0 = m0 / hpg, items = (min(RT, p.M - m0) / hpg) * half;
+            // pair k: elements (k, k + half) in the half-split style, (2k, 2k + 1) interleaved
+            const int s0 = pe.style == 0 ? 1 : 2, o1 = pe.style == 0 ? half : 1;
+            for (int it = slot * 128 + (warp & 3) * 32 + lane; it < items; it += slots * 128) {
+                const int k = it % half, bi = tok0 + it / half;  // bi = b q_len + i
+                const int b = bi / pe.q_len, i = bi - b * pe.q_len;
+                float cs, sn;
+                rope_cos_sin(static_cast<int64_t>(__ldg(pe.kv_len + b)) - pe.q_len + i, pe.turns.f[k], &cs, &sn);
+                const int64_t row0 = static_cast<int64_t>(bi) * p.blk + static_cast<int64_t>(g) * hpg;
+                const int c0 = s0 * k, c1 = o1 + s0 * k;
+                for (int h0 = 0; h0 < hpg; h0 += 4) {
+                    uint16_t x0[4], x1[4];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u)
+                        if (h0 + u < hpg) {
+                            const uint16_t *src = pe.rope_src + (row0 + h0 + u) * pe.d_rope;
+                            x0[u] = __ldg(src + c0);
+                            x1[u] = __ldg(src + c1);
+                        }
+#pragma unroll
+                    for (int u = 0; u < 4; ++u)
+                        if (h0 + u < hpg) {
+                            const float a0 = __uint_as_float(static_cast<uint32_t>(x0[u]) << 16);
+                            const float a1 = __uint_as_float(static_cast<uint32_t>(x1[u]) << 16);
+                            uint16_t *dst = static_cast<uint16_t *>(p.C) + (row0 + h0 + u) * p.ldc + pe.rank;
+                            dst[c0] = __bfloat16_as_ushort(__float2bfloat16_rn(a0 * cs - a1 * sn));
+                            dst[c1] = __bfloat16_as_ushort(__float2bfloat16_rn(a1 * cs + a0 * sn));
+                        }
+                }
+            }
+        }
         // ---- epilogue: warp w reads TMEM lanes 32 (w % 4) .. + 31
         const bool ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(&bars.done), 0, lim));
         if (!ok) {
@@ -526,12 +573,20 @@ int ring_stages(int K, size_t *smem)
 }
 
 template <int BN, bool NMAJ, bool AF32>
-cudaError_t launch_tc(const GroupGemm &p, cudaStream_t st)
+cudaError_t launch_tc(const GroupGemm &p, cudaStream_t st, const ProjEpi *rope = nullptr)
 {
     cudaError_t e = get_encoder();
     if (e != cudaSuccess) return e;
     if (p.hpg < 1 || p.hpg > 128 || p.M % p.hpg) return cudaErrorInvalidValue;
-    const int rblk = rows_per_tile(p);
+    int rblk = rows_per_tile(p);
+    const int ntiles = (p.N + BN - 1) / BN;
+    const int nk = (p.K + 63) / 64;
+    auto tiles_for = [&](int rb) { return static_cast<int64_t>((p.M / p.hpg + rb - 1) / rb) * ntiles * p.G; };
+    // A grid too small to spread over the SMs and K too short to split (the
+    // split below wants deep K): shorter row tiles instead, each CTA
+    // re-reading its (small) weight tile from L2
+    if (nk < 8)
+        while (tiles_for(rblk) < 64 && rblk > 1 && rblk * p.hpg > 16) rblk = (rblk + 1) / 2;
     CUtensorMap ma, mb;
     if (!encode_a(p, rblk, AF32, &ma)) return cudaErrorInvalidValue;
     if (NMAJ) {  // [G K rows][N columns], 64 x 64 boxes
@@ -546,12 +601,11 @@ cudaError_t launch_tc(const GroupGemm &p, cudaStream_t st)
         return cudaErrorInvalidValue;
     }
     const int rt = rblk * p.hpg;
-    const int mtiles = (p.M + rt - 1) / rt, ntiles = (p.N + BN - 1) / BN;
+    const int mtiles = (p.M + rt - 1) / rt;
     // Split K over a cluster when the tiles are short (<= 64 rows: a small
     // batch), K is deep (>= 8 chunks) and the tiles alone would leave most SMs
     // idle: up to 4 ways, at least two chunks each, with a ring of at most 4
     // stages so that two CTAs share an SM and the split grid runs in one wave.
-    const int nk = (p.K + 63) / 64;
     const int64_t tiles = static_cast<int64_t>(mtiles) * ntiles * p.G;
     int ks = 1;
     if (rt <= 64 && nk >= 8)
@@ -575,7 +629,7 @@ cudaError_t launch_tc(const GroupGemm &p, cudaStream_t st)
     dim3 grid(mtiles * ks, ntiles, p.G);
     ProjEpi none{};
     return launch_dependent(gemm_tc_kernel<BN, NMAJ, AF32, false>, grid, dim3(kGemmThreads), smem, st, ks, q, ma, mb,
-                            mb, mb, none);
+                            mb, mb, rope ? *rope : none);
 }
 
 // The projection: h [M = batch n_new, hidden] against W^DKV (rank rows), W^KR
@@ -640,6 +694,25 @@ cudaError_t launch_proj(const mla_dims &d, const CacheView &c, int batch, int n_
 }
 
 }  // namespace
+
+// The absorption GEMM with the positional-query rotation in its epilogue
+// warps (N-major W_UK, bf16 q_nope).
+cudaError_t launch_absorb_gemm(const GroupGemm &p, const mla_dims &d, const void *q_pe, const int32_t *kv_len,
+                               int q_len, cudaStream_t st)
+{
+    if (p.M <= 0 || p.N <= 0 || p.G <= 0) return cudaSuccess;
+    ProjEpi r{};
+    r.rope_src = static_cast<const uint16_t *>(q_pe);
+    r.kv_len = kv_len;
+    r.q_len = q_len;
+    r.heads = d.num_heads;
+    r.rank = d.rank;
+    r.d_rope = d.d_rope;
+    r.style = d.rope_style;
+    r.turns = rope_turns(d.d_rope, d.rope_base);
+    const bool narrow = p.N <= 64 || p.M <= 32;
+    return narrow ? launch_tc<64, true, false>(p, st, &r) : launch_tc<128, true, false>(p, st, &r);
+}
 
 cudaError_t launch_group_gemm(const GroupGemm &p, cudaStream_t st)
 {

@@ -86,6 +86,10 @@ struct GroupGemm {
     int stages, rblk, ksplit;  // set by the launcher
 };
 cudaError_t launch_group_gemm(const GroupGemm &p, cudaStream_t st);
+// The absorption GEMM (N-major W_UK, bf16 A) that also writes the rotated
+// positional query into columns [rank, rank + d_rope) of its output rows.
+cudaError_t launch_absorb_gemm(const GroupGemm &p, const mla_dims &d, const void *q_pe, const int32_t *kv_len,
+                               int q_len, cudaStream_t st);
 
 // Projection of the step's hidden states (mla_project_append): one GEMM of
 // h [batch * n_new, hidden] with the three weights side by side, whose
