@@ -191,7 +191,7 @@ __device__ void proj_epilogue(const GroupGemm &p, const ProjEpi &e, uint32_t t_l
 // of hpg rows, i.e. RT = R hpg <= 128 rows.  A bf16 A box lands directly in
 // the 128B-swizzled K-major layout the MMA reads; an fp32 A (o_lat) lands as
 // two 32-column boxes in a staging tile, which four warps convert to bf16.
-constexpr int kStages = 8;  // most ring stages; fewer when K is short or shared memory runs out
+constexpr int kStages = 16;  // most ring stages; fewer when K is short or shared memory runs out
 constexpr int kGemmThreads = 192;  // warp 0 TMA, warp 1 MMA, warps 2..5 convert / epilogue
 
 struct __align__(8) GemmBars {
@@ -233,8 +233,14 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
     const int kz = blockIdx.x % ks;                      // this CTA's share: chunks [c_begin, c_end)
     const int c_begin = kz * nk / ks, nkl = (kz + 1) * nk / ks - c_begin;
     const int NS = p.stages;                             // ring stages (<= kStages)
+    // A stages sit a_stride apart: a full tile, or for a bf16 A of RT <= 64
+    // rows just those rows (rounded to 8).  The M = 128 MMA still reads 128
+    // rows from its stage base: the rows past RT come from the next stages or
+    // the B ring (inside the allocation), land in accumulator rows >= RT and
+    // are never stored.
+    const int AS = (AF32 || PROJ) ? kABytes : p.a_stride;
     unsigned char *sa = smem;                            // NS x A tile
-    unsigned char *sb = sa + NS * kABytes;               // NS x B tile
+    unsigned char *sb = sa + NS * AS;                    // NS x B tile
     unsigned char *sr = sb + NS * kBBytes;               // NS x raw fp32 A (AF32)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int R = p.rblk, RT = R * p.hpg;                // row blocks and rows per tile (<= 128)
@@ -311,7 +317,7 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
                     tma_load_4d(rdst, &map_a, 64 * c, 0, g, mt * R, rb);
                     tma_load_4d(rdst + 128 * 128, &map_a, 64 * c + 32, 0, g, mt * R, rb);
                 } else {
-                    tma_load_4d(smem_u32(sa + s * kABytes), &map_a, 64 * c, 0, g, mt * R, fb);
+                    tma_load_4d(smem_u32(sa + s * AS), &map_a, 64 * c, 0, g, mt * R, fb);
                 }
             }
             __syncwarp();
@@ -332,7 +338,7 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
                                              (!AF32 || mbar_wait(smem_u32(&bars.conv_done[s]), par, lim)));
             if (!ok) break;
             tc::fence_after_sync();
-            const uint32_t a_base = smem_u32(sa + s * kABytes), b_base = smem_u32(sb + s * kBBytes);
+            const uint32_t a_base = smem_u32(sa + s * AS), b_base = smem_u32(sb + s * kBBytes);
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk) {
                 const uint32_t b_addr = NMAJ ? b_base + kk * 16 * 128 : b_base + kk * 32;
@@ -355,7 +361,7 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
                 }
                 const uint4 *src0 = reinterpret_cast<const uint4 *>(sr + s * kRawBytes + r * 128);
                 const uint4 *src1 = reinterpret_cast<const uint4 *>(sr + s * kRawBytes + 128 * 128 + r * 128);
-                uint4 *dst = reinterpret_cast<uint4 *>(sa + s * kABytes + r * 128);
+                uint4 *dst = reinterpret_cast<uint4 *>(sa + s * AS + r * 128);
 #pragma unroll
                 for (int j = 0; j < 8; ++j) {
                     // bf16 16-byte chunk j = fp32 chunks 2j, 2j + 1 (of box j / 4)
@@ -610,12 +616,39 @@ cudaError_t launch_tc(const GroupGemm &p, cudaStream_t st, const ProjEpi *rope =
     int ks = 1;
     if (rt <= 64 && nk >= 8)
         while (ks < 4 && tiles * ks * 2 <= (AF32 ? 152 : 2 * 152) && nk >= 4 * ks) ks *= 2;  // fp32 A: one CTA per SM
+    // Full 128-row tiles that would fill fewer than half the SMs (a mid-size
+    // batch against a wide weight): split K as well, one CTA per SM, at least
+    // eight chunks per share, the partials (128 rows x BN / ks columns from
+    // each rank) pushed into the ring.  (Not for an fp32 A: there the
+    // reduction cost as much as the split saved.)
+    const bool wide_split = rt > 64 && !AF32 && nk >= 16 && tiles * 2 <= 152;
+    if (wide_split)
+        while (ks < 4 && tiles * ks * 2 <= 152 && nk >= 8 * ks) ks *= 2;
     size_t smem = 0;
     GroupGemm q = p;
-    q.stages = ring_stages<BN, AF32>((nk + ks - 1) / ks * 64, &smem);
-    if (ks > 1 && q.stages > 4) {
-        q.stages = 4;
-        smem = 1024 + 4 * (128 * 128 + BN * 128 + (AF32 ? 2 * 128 * 128 : 0));
+    q.a_stride = 128 * 128;
+    if (!AF32 && rt <= 64) {
+        // short bf16 A tiles: stages of RT rows (rounded to 8), so that the ring
+        // holds many more weight chunks -- with a split, all of a CTA's chunks
+        // at two CTAs per SM -- and the weights stream with more bytes in flight
+        q.a_stride = (rt + 7) / 8 * 8 * 128;
+        const int nkl = (nk + ks - 1) / ks;
+        const size_t per_stage = static_cast<size_t>(q.a_stride) + BN * 128;
+        const size_t budget = ks > 1 ? 110 * 1024 : 192 * 1024;
+        int ns = static_cast<int>(budget / per_stage);
+        ns = ns > kStages ? kStages : ns;
+        ns = ns > nkl ? nkl : ns;
+        q.stages = ns < 1 ? 1 : ns;
+        // the last stage's MMA reads a full 128-row window from its base
+        const size_t ring = static_cast<size_t>(q.stages) * per_stage;
+        const size_t window = static_cast<size_t>(q.stages - 1) * q.a_stride + 128 * 128;
+        smem = 1024 + (ring > window ? ring : window);
+    } else {
+        q.stages = ring_stages<BN, AF32>((nk + ks - 1) / ks * 64, &smem);
+        if (ks > 1 && !wide_split && q.stages > 4) {
+            q.stages = 4;
+            smem = 1024 + 4 * (128 * 128 + BN * 128 + (AF32 ? 2 * 128 * 128 : 0));
+        }
     }
     q.rblk = rblk;
     q.ksplit = ks;

@@ -84,6 +84,7 @@ struct GroupGemm {
     int64_t ldc;
     unsigned *status;
     int stages, rblk, ksplit;  // set by the launcher
+    int a_stride;              // bytes between A ring stages (set by the launcher)
 };
 cudaError_t launch_group_gemm(const GroupGemm &p, cudaStream_t st);
 // The absorption GEMM (N-major W_UK, bf16 A) that also writes the rotated
