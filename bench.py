@@ -35,6 +35,7 @@ sys.path.insert(0, ROOT)
 
 DEFAULT_WORKLOAD = "qwen05b_b16_h14_r256_t2048"
 METRIC = "MLA decode-attn μs/step and latent-cache HBM GB/s (% of GB300 peak), 1 GPU"
+NOMINAL_HBM_GBS = 8000.0  # the ~8 TB/s HBM3e figure the attention target is also quoted against
 
 
 def parse_args(argv=None):
@@ -208,14 +209,17 @@ def run_ours(args, rank, world, local):
         clocks.start()
         barrier(world)
         torch.cuda.synchronize(dev)
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
+        # one event before each step and one after the last: the first and the
+        # last bracket the K steps, the ones between give each step's time
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+        ev[0].record(stream)
         for i in range(args.steps):
             one(i)
-        e1.record(stream)
+            ev[i + 1].record(stream)
         torch.cuda.synchronize(dev)
         barrier(world)
-        elapsed_ms = e0.elapsed_time(e1)
+        elapsed_ms = ev[0].elapsed_time(ev[-1])
+        step_ms = sorted(ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps))
         # keep the GPU loaded for at least ~1.5 s so the clock samples cover a busy GPU
         t_end = time.time() + max(0.0, 1.5 - elapsed_ms / 1e3)
         i = args.steps
@@ -307,6 +311,17 @@ def run_ours(args, rank, world, local):
     attn_avg_ms = sum(attn_ms) / len(attn_ms)
     peaks = load_peaks()
     achieved = cache_bytes / (attn_avg_ms * 1e-3) / 1e9
+    # algorithmic flops of the attention core: per query (b, i, head) with
+    # kv_b - q + i + 1 visible keys, 2 (r + d_rope) per key for the scores and 2 r
+    # for P C
+    kv = [int(x) for x in w.kv_len.tolist()]
+    keys = sum(k - shape.q_len + i + 1 for k in kv for i in range(shape.q_len)) * shape.num_heads
+    attn_flops = float(keys) * (2 * (shape.rank + shape.d_rope) + 2 * shape.rank)
+    attn_tflops = attn_flops / (attn_avg_ms * 1e-3) / 1e12
+    t_floor = max(cache_bytes / (peaks["hbm_gbs"] * 1e9), attn_flops / (peaks["bf16_tflops"] * 1e12))
+
+    def pct(q):
+        return round(step_ms[min(len(step_ms) - 1, int(q * len(step_ms)))] * 1e3, 3)
     launches_per_step = 1 + 1 + 1 + 1 + (2 if shape.hidden else 1)  # append, absorb, attention, combine, W_UV (+ W_O)
     line = {
         "metric": METRIC,
@@ -318,6 +333,7 @@ def run_ours(args, rank, world, local):
         "ms_per_step": round(ms_step, 6),
         "us_per_step": round(ms_step * 1e3, 3),
         "attn_us_per_launch": round(attn_avg_ms * 1e3, 3),
+        "attn_combine_us": gqa.get("mla_us") if isinstance(gqa, dict) else None,
         "queries_per_s": round(world * shape.batch * shape.q_len / (ms_step * 1e-3), 1),
         "higher_is_better": True,
         "scaling": "weak",
@@ -340,7 +356,12 @@ def run_ours(args, rank, world, local):
             "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": attn_traffic(shape.name),
             "peak_source": peaks["source"], "kernel": "mla_decode_attn",
             "bytes_per_launch": cache_bytes,
+            "flops_per_launch": attn_flops, "achieved_tflops": round(attn_tflops, 1),
+            "tensor_frac": round(attn_tflops / peaks["bf16_tflops"], 4),
+            "ridge_frac": round(t_floor / (attn_avg_ms * 1e-3), 4),
+            "nominal_gbs": NOMINAL_HBM_GBS, "nominal_frac": round(achieved / NOMINAL_HBM_GBS, 4),
         },
+        "step_us_dist": {"p10": pct(0.1), "p50": pct(0.5), "p90": pct(0.9)},
         "clocks": clocks.summary(),
         "e2e": {"value": round(total_bytes / (max_e2e * 1e-3) / 1e9, 2), "unit": "GB/s",
                 "us_per_step": round(max_e2e / args.steps * 1e3, 3),
