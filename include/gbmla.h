@@ -118,8 +118,11 @@ typedef struct mla_cache {
 /* Sizes of the two partial buffers mla_decode_attn writes for this problem,
  * and the number of partitions S it will use: num_splits > 0 is taken as
  * given, 0 picks S from the device's SM count (the same rule every call of
- * this library applies).  max_kv_len bounds every kv_len[b].  Any output
- * pointer may be NULL. */
+ * this library applies): one partition per SM (per group of SMs sharing a
+ * tile); when that leaves at most four tiles per partition (the tiles counted
+ * as batch x ceil(max_kv_len / MLA_SPLIT_TILE)), the fewest partitions that
+ * keep the same most tiles per partition.
+ * max_kv_len bounds every kv_len[b].  Any output pointer may be NULL. */
 mla_status mla_workspace_size(const mla_dims *dims, int32_t batch, int32_t q_len, int32_t max_kv_len,
                               int32_t num_splits, size_t *o_part_bytes, size_t *lse_part_bytes,
                               int32_t *num_splits_used);
