@@ -12,7 +12,9 @@
 // chunks again, from L2) the value products, so that the softmax of tile t
 // overlaps QK(t+1) and PV(t-1).  With two query groups (160 query rows) the
 // two CTAs form a cluster and every cache box is multicast to both, so each
-// byte leaves L2 once per pass.
+// byte leaves L2 once per pass.  A sequence's last, partial tile issues only
+// the value products of its 16-token steps that hold cached rows; the PV warp
+// clears the rows past the end inside the last such step itself.
 //
 // Warp roles (512 threads): warps 0 and 3 = TMA producers (QK ring and query
 // boxes; PV ring), warp 1 = QK MMA issuer and TMEM owner, warp 2 = PV MMA
@@ -83,10 +85,6 @@ struct __align__(8) Bars {
     uint64_t s_full[2], s_free[2];
     uint64_t p_full[2], pv_done[2];  // per P buffer (t % NP): P(t) published / PV(t) completed
     uint64_t o_free, drain_qk, drain_pv;
-    // Tail tile handshake per r-chunk m: the PV warp (which waits on its
-    // ring in strict order) reports that chunks 2m, 2m+1 landed (zready);
-    // the softmax warps clear their rows past the end (zdone).
-    uint64_t zready[4], zdone[4];
 };
 
 template <int N>
@@ -389,7 +387,6 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
     float l_part[KOWN][16];
     int b_cur = -1;
     int64_t t_last = -1;
-    int n_tail = 0;  // tail tiles handled so far (phase of zready / zdone)
     const int cc = c.tid - kSoftmaxBase;
     Walk w;
     w.init(a.kv_len, a.batch, a.q_len, a.max_kv, c.t_begin, c.t_end);
@@ -537,29 +534,6 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
         __syncwarp();
         if (c.lane == 0) tc::mbar_arrive(smem_u32(&bars.p_full[t % kPBufs<N>]));
         if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(9, t);
-        // ---- tail tile: rows past the sequence end in the PV copy of the
-        // latent chunks are cleared, so stale or uninitialised bytes never meet
-        // a zero weight.  P is already published; the MMA warp reports each
-        // landed pair (zready) and waits for it to be cleared (zdone), so every
-        // wait here is on the next phase of its barrier.
-        if (last && kv - j * kTile < kTile) {
-            const int64_t g0 = static_cast<int64_t>(c.ncc) * t;  // first PV-ring chunk of tile t
-            for (int m = 0; m < c.nrc; ++m) {
-                sm_wait<N>(c, a, ss, &bars.zready[m], static_cast<uint32_t>(n_tail & 1));
-                if (pos >= kv) {
-                    for (int k = 0; k < 2; ++k) {
-                        const int slot = static_cast<int>((g0 + 2 * m + k) % c.cs);
-                        // three warps share a quarter's rows: 16-byte pieces half, half+3, ...
-                        uint4 *dst = reinterpret_cast<uint4 *>(c.ring + slot * kChunkBytes + c.tok * 128);
-                        for (int q = c.half; q < 8; q += 3) dst[q] = make_uint4(0, 0, 0, 0);
-                    }
-                }
-                tc::fence_proxy_async_smem();
-                __syncwarp();
-                if (c.lane == 0) tc::mbar_arrive(smem_u32(&bars.zdone[m]));
-            }
-            ++n_tail;
-        }
     }
     named_sync_softmax();
     if (b_cur >= 0 && !ss.sm_fail) sm_epilogue<N, KOWN>(c, a, ss, bars, l_part, b_cur, t_last);
@@ -614,10 +588,6 @@ __global__ void __maxnreg__(128)
         mbar_init(&bars.o_free, kSoftmaxWarps);
         mbar_init(&bars.drain_qk, 1);
         mbar_init(&bars.drain_pv, 1);
-        for (int i = 0; i < 4; ++i) {
-            mbar_init(&bars.zready[i], 1);
-            mbar_init(&bars.zdone[i], kSoftmaxWarps);
-        }
 #ifdef GBMLA_TRACE
         s_trace_count = 0;
         s_sm_wait_cyc = 0;
@@ -861,7 +831,7 @@ __global__ void __maxnreg__(128)
             } else {
                 const uint32_t id_pv = tc::idesc_bf16_f32(128, N, true, true);
                 const uint32_t ring_base = smem_u32(ring_b);
-                int seg = -1, n_tail = 0;
+                int seg = -1;
                 for (int t = 0; t < n_items && ok; ++t, w.next()) {
                     if (any_abort()) break;
                     if (!wait(&bars.p_full[t % kPBufs<N>], (t / kPBufs<N>) & 1)) break;
@@ -872,23 +842,34 @@ __global__ void __maxnreg__(128)
                         if (seg >= 1 && !wait(&bars.o_free, (seg - 1) & 1)) break;
                         first_pv = true;
                     }
-                    // a sequence's last, partial tile: its rows past the end are cleared
-                    // by the softmax warps, pair by pair, before PV reads them
-                    const bool tail = w.last() && a.kv_len[w.b] - w.tile() * kTile < kTile;
+                    // A sequence's last, partial tile of v rows: only the 16-token
+                    // steps holding rows < v are issued, and in the last of them the
+                    // rows v .. v16 - 1 of both chunks are cleared here first, so that
+                    // stale or uninitialised bytes never meet a zero weight (0 x NaN
+                    // is NaN).  Rows past v16 are never read.
+                    const int v = a.kv_len[w.b] - w.tile() * kTile;
+                    const bool tail = w.last() && v < kTile;
+                    const int v16 = tail ? (v + 15) / 16 * 16 : kTile;
                     for (int m = 0; m < nrc && ok; ++m) {
                         // chunks 2m, 2m+1 sit in adjacent slots (CB and ncc are even)
                         const int s0 = rp.slot;
                         if (!wait(&bars.pv_full[s0], rp.round & 1) || !wait(&bars.pv_full[s0 + 1], rp.round & 1)) break;
-                        if (tail) {
-                            tc::mbar_arrive_elect(smem_u32(&bars.zready[m]));
-                            if (!wait(&bars.zdone[m], n_tail & 1)) break;
-                        }
                         tc::fence_after_sync();
+                        if (v16 > v) {
+                            const int nz = (v16 - v) * 8;  // 16-byte pieces per chunk
+                            for (int idx = lane; idx < 2 * nz; idx += 32) {
+                                const int k = idx / nz, r = idx - k * nz;
+                                uint4 *dst = reinterpret_cast<uint4 *>(ring_b + (s0 + k) * kChunkBytes +
+                                                                       (v + r / 8) * 128) + r % 8;
+                                *dst = make_uint4(0, 0, 0, 0);
+                            }
+                            tc::fence_proxy_async_smem();
+                            __syncwarp();
+                        }
                         const uint32_t cb = ring_base + s0 * kChunkBytes;
                         const uint32_t pb = p_base + (t % kPBufs<N>) * (N / 16) * (kTile * 32);
                         const uint32_t d_o = tmem + o_col0 + m * N;
-#pragma unroll
-                        for (int kk = 0; kk < kTile / 16; ++kk)
+                        for (int kk = 0; kk < v16 / 16; ++kk)
                             tc::mma_bf16_elect(d_o, with_addr(dc, cb + kk * 16 * 128),
                                                with_addr(dp, pb + kk * 16 * 32), id_pv,
                                                (first_pv && kk == 0) ? 0u : 1u);
@@ -900,7 +881,6 @@ __global__ void __maxnreg__(128)
                     if (!ok) break;
                     tc::commit_elect(smem_u32(&bars.pv_done[t % kPBufs<N>]));
                     if (lane == 0) GBMLA_TRACE_EVENT(5, t);
-                    if (tail) ++n_tail;
                 }
             }
             if (!ok && lane == 0) {
