@@ -26,6 +26,8 @@
 #include <math.h>
 #include <stdlib.h>
 
+#include <type_traits>
+
 #include "common.cuh"
 #include "internal.h"
 #include "tc.cuh"
@@ -46,25 +48,50 @@ constexpr int kThreads = kSoftmaxBase + 32 * kSoftmaxWarps;
 template <int N>
 constexpr int kPBufs = N >= 80 ? 1 : 2;
 
-// Optional event trace of the first CTA (compiled only with -DGBMLA_TRACE):
-// (globaltimer ns, event code, argument) triples in a caller buffer, set by
-// mla_debug_trace().  Used to read the per-tile timeline of the roles.
+// O^T buffers in TMEM: two where they fit beside the two S^T buffers (2N + 2 x 4N
+// columns <= 512, i.e. N <= 48), so that a sequence's value products start in
+// one while the previous sequence's partial drains from the other; else one.
+template <int N>
+constexpr int kOBufs = 10 * N <= 512 ? 2 : 1;
+template <int N>
+constexpr uint32_t kTmemCols = (2 * N + kOBufs<N> * 4 * N) <= 128 ? 128u
+                               : (2 * N + kOBufs<N> * 4 * N) <= 256 ? 256u : 512u;
+
+// Optional event trace (compiled only with -DGBMLA_TRACE): (globaltimer ns,
+// event code, argument) triples in a caller buffer of 2 cap entries (two
+// 64-bit words each), set by mla_debug_trace(buf, cap): entries 0 .. cap - 1
+// hold the role timeline of one CTA (mla_debug_trace_cta picks it, default
+// 0), entries cap .. 2 cap - 1 every CTA's start, end and tile range.
 #ifdef GBMLA_TRACE
 __device__ unsigned long long *g_trace_buf;
 __device__ unsigned g_trace_count;
 __device__ unsigned g_trace_cap;
+__device__ unsigned g_trace_which;  // the CTA (y * gridDim.x + x) whose roles are traced
 __shared__ unsigned s_trace_count;  // events of this CTA (a shared-memory atomic keeps the probe cheap)
 __device__ __forceinline__ void trace_event(int code, int64_t arg)
 {
-    if (blockIdx.x != 0 || blockIdx.y != 0 || g_trace_buf == nullptr) return;
+    if (blockIdx.y * gridDim.x + blockIdx.x != g_trace_which || g_trace_buf == nullptr) return;
     const unsigned i = atomicAdd(&s_trace_count, 1u);
     if (i >= g_trace_cap) return;
     g_trace_buf[2 * i] = global_ns();
     g_trace_buf[2 * i + 1] = (static_cast<unsigned long long>(code) << 48) | (static_cast<unsigned long long>(arg) & 0xffffffffffffull);
 }
+// Every CTA: (time, code, argument) of its start, end and tile range, in
+// entries cap .. 2 cap - 1 of the same buffer.
+__device__ __forceinline__ void trace_cta(int code, int64_t arg)
+{
+    if (g_trace_buf == nullptr) return;
+    const unsigned i = atomicAdd(&g_trace_count, 1u);
+    if (i >= g_trace_cap) return;
+    g_trace_buf[2 * (g_trace_cap + i)] = global_ns();
+    g_trace_buf[2 * (g_trace_cap + i) + 1] =
+        (static_cast<unsigned long long>(code) << 48) | (static_cast<unsigned long long>(arg) & 0xffffffffffffull);
+}
 #define GBMLA_TRACE_EVENT(code, arg) trace_event((code), (arg))
+#define GBMLA_TRACE_CTA(code, arg) trace_cta((code), (arg))
 #else
 #define GBMLA_TRACE_EVENT(code, arg) ((void)0)
+#define GBMLA_TRACE_CTA(code, arg) ((void)0)
 #endif
 
 struct TcArgs {
@@ -84,15 +111,34 @@ struct __align__(8) Bars {
     uint64_t q_full, q_free;
     uint64_t s_full[2], s_free[2];
     uint64_t p_full[2], pv_done[2];  // per P buffer (t % NP): P(t) published / PV(t) completed
-    uint64_t o_free, drain_qk, drain_pv;
+    uint64_t o_free, drain_qk, drain_pv;  // o_free: O^T buffer 0 drained
 };
+
+// With two O^T buffers, the barrier of the second.  (A kernel with one buffer
+// keeps the plain layout: one more member there changed its register
+// allocation enough to spill.)
+struct BarsO2 : Bars {
+    uint64_t o_free1;
+};
+template <int N>
+using BarsT = std::conditional_t<kOBufs<N> == 2, BarsO2, Bars>;
+
+template <class B>
+__device__ __forceinline__ uint64_t *o_free_bar(B &b, int i)
+{
+    if constexpr (std::is_same_v<B, BarsO2>)
+        return i ? &b.o_free1 : &b.o_free;
+    else
+        return &b.o_free;
+}
 
 template <int N>
 struct Shared {
     float red[4][N];   // per TMEM-quadrant column partials
     float m_used[N];   // exponent base of each query column (log2 domain)
     float alpha[N];    // rescale factor of the current tile
-    float lsum[N];     // softmax denominators at the epilogue
+    float lsum[N];     // softmax denominators at the epilogue (one O^T buffer)
+    float inv_l[N];    // 1 / softmax denominator of the last closed sequence (two buffers)
     int lim[N];        // last visible position of each column (-1: padding column)
     int need_max;
     int any_rescale;
@@ -129,6 +175,7 @@ struct Walk {
     __device__ int tile() const { return static_cast<int>(t - seq_start); }
     __device__ bool first() const { return t == t_begin || t == seq_start; }
     __device__ bool last() const { return t + 1 == t_end || t + 1 == seq_start + nb; }
+    __device__ bool last_of_partition() const { return t + 1 == t_end; }
     __device__ void next()
     {
         ++t;
@@ -321,7 +368,7 @@ __device__ __forceinline__ void sm_block_max(const SmCtx &c, const TcArgs &a, Sh
 }
 
 // Normalised partial output and log-sum-exp of sequence b, whose last tile
-// in this partition was t_end_seg.
+// in this partition was t_end_seg, in one step (one O^T buffer).
 template <int N, int KOWN>
 __device__ __forceinline__ void sm_epilogue(const SmCtx &c, const TcArgs &a, Shared<N> &ss, Bars &bars,
                                             float (&l_part)[KOWN][16], int b, int64_t t_end_seg)
@@ -379,14 +426,82 @@ __device__ __forceinline__ void sm_epilogue(const SmCtx &c, const TcArgs &a, Sha
     if (c.lane == 0) tc::mbar_arrive(smem_u32(&bars.o_free));
 }
 
+// Closing a sequence b of this partition (no wait on its value products):
+// its softmax denominators (1 / l kept for the drain) and its log-sum-exp.
+template <int N, int KOWN>
+__device__ __forceinline__ void sm_close(const SmCtx &c, const TcArgs &a, Shared<N> &ss, float (&l_part)[KOWN][16],
+                                         int b)
+{
+#pragma unroll
+    for (int ob = 0; ob < KOWN; ++ob) {
+        if (ob < c.n_own) {
+            const int cb = c.half + 3 * ob;
+            float v[16];
+#pragma unroll
+            for (int e = 0; e < 16; ++e) v[e] = l_part[ob][e];
+            const float ls = reduce16<false>(v, c.lane);
+            if (c.lane < 16) ss.red[c.quarter][cb * 16 + c.lane] = ls;
+        }
+    }
+    named_sync_softmax();
+    const int cc = c.tid - kSoftmaxBase;
+    if (cc < N) {
+        const float l = ss.red[0][cc] + ss.red[1][cc] + ss.red[2][cc] + ss.red[3][cc];
+        ss.inv_l[cc] = l > 0.f ? 1.f / l : 0.f;
+        const int row = c.group * N + cc;
+        if (row < a.rows) {
+            const int64_t slot = static_cast<int64_t>(b) + c.part;
+            a.lse_part[slot * a.rows + row] = l > 0.f ? (ss.m_used[cc] + log2f(l)) * 0.69314718055994531f : -INFINITY;
+        }
+    }
+    named_sync_softmax();  // inv_l is complete and red is free again
+}
+
+// The normalised partial output of sequence b (closed by sm_close), whose
+// last tile here was t_end_seg, from O^T buffer obuf; then the buffer is free.
+template <int N, int KOWN>
+__device__ __forceinline__ void sm_drain(const SmCtx &c, const TcArgs &a, Shared<N> &ss, BarsT<N> &bars, int b,
+                                         int64_t t_end_seg, int obuf)
+{
+    sm_wait<N>(c, a, ss, &bars.pv_done[t_end_seg % kPBufs<N>], static_cast<uint32_t>((t_end_seg / kPBufs<N>) & 1));
+    named_sync_softmax();
+    if (ss.sm_fail) return;
+    tc::fence_after_sync();
+    const int64_t slot = static_cast<int64_t>(b) + c.part;
+    const int valid_cols = a.rows - c.group * N;  // columns past it are padding
+    float *out = a.o_part + (slot * a.rows + c.group * N) * a.rank + c.tok;
+    const uint32_t o_col = c.o_col0 + static_cast<uint32_t>(obuf * 4 * N);
+    for (int m = 0; m < c.nrc; ++m) {
+#pragma unroll
+        for (int ob = 0; ob < KOWN; ++ob) {
+            if (ob < c.n_own) {
+                const int cb = c.half + 3 * ob;
+                float o[16];
+                tmem_ld16(c.tmem + c.lane_base + o_col + m * N + cb * 16, o);
+#pragma unroll
+                for (int e = 0; e < 16; ++e) {
+                    const int col = cb * 16 + e;
+                    if (col < valid_cols) out[col * a.rank + m * 128] = o[e] * ss.inv_l[col];
+                }
+            }
+        }
+    }
+    tc::fence_before_sync();
+    __syncwarp();
+    if (c.lane == 0) tc::mbar_arrive(smem_u32(o_free_bar(bars, obuf)));
+}
+
 template <int N>
-__device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Shared<N> &ss, Bars &bars)
+__device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Shared<N> &ss, BarsT<N> &bars)
 {
     constexpr int NB = N / 16;
     constexpr int KOWN = (NB + 2) / 3;
     float l_part[KOWN][16];
     int b_cur = -1;
-    int64_t t_last = -1;
+    int u = -1;  // sequences begun here (the PV warp counts the same ones)
+    int64_t t_prev = -1;  // the previous tile (one O^T buffer: the drain runs at the next sequence's first tile)
+    // a closed sequence whose drain waits for the next sequence's first P (two O^T buffers)
+    int d_b = -1, d_t = -1;
     const int cc = c.tid - kSoftmaxBase;
     Walk w;
     w.init(a.kv_len, a.batch, a.q_len, a.max_kv, c.t_begin, c.t_end);
@@ -401,11 +516,14 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
         if (ss.sm_fail) break;
         tc::fence_after_sync();
         if (first) {
-            if (b_cur >= 0) {
-                sm_epilogue<N, KOWN>(c, a, ss, bars, l_part, b_cur, t_last);
-                if (ss.sm_fail) break;
+            if constexpr (kOBufs<N> == 1) {
+                if (b_cur >= 0) {
+                    sm_epilogue<N, KOWN>(c, a, ss, bars, l_part, b_cur, t_prev);
+                    if (ss.sm_fail) break;
+                }
             }
             b_cur = b;
+            ++u;
 #pragma unroll
             for (int ob = 0; ob < KOWN; ++ob)
 #pragma unroll
@@ -416,7 +534,7 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
             }
             named_sync_softmax();
         }
-        t_last = t;
+        t_prev = t;
         const int pos = j * kTile + c.tok;
         // the mask matters only where a token lies past the earliest query's last key
         const bool need_mask = j * kTile + kTile - 1 > kv - a.q_len;
@@ -492,7 +610,8 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
                             l_part[ob][e] *= al[e];
                         }
                         for (int m = 0; m < c.nrc; ++m) {
-                            const uint32_t ta = c.tmem + c.lane_base + c.o_col0 + m * N + cb * 16;
+                            const uint32_t ta = c.tmem + c.lane_base + c.o_col0 +
+                                                static_cast<uint32_t>((u % kOBufs<N>) * 4 * N + m * N + cb * 16);
                             float o[16];
                             tmem_ld16(ta, o);
 #pragma unroll
@@ -534,9 +653,48 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
         __syncwarp();
         if (c.lane == 0) tc::mbar_arrive(smem_u32(&bars.p_full[t % kPBufs<N>]));
         if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(9, t);
+        if constexpr (kOBufs<N> == 2) {
+            // Due now, in this order: the previous sequence's drain (deferred
+            // until this first P was out, so that it overlaps this tile's value
+            // products in the other O^T buffer); then, on a sequence's last
+            // tile, its close -- and at the partition's end its drain.
+#pragma unroll 1
+            for (int k = 0; k < 2; ++k) {
+                int db = -1, dt = 0, dbuf = 0;
+                if (k == 0 && d_b >= 0) {
+                    db = d_b;
+                    dt = d_t;
+                    dbuf = (u - 1) & 1;
+                    d_b = -1;
+                }
+                if (k == 1 && last) {
+                    named_sync_softmax();
+                    sm_close<N, KOWN>(c, a, ss, l_part, b_cur);
+                    if (!w.last_of_partition()) {
+                        d_b = b_cur;
+                        d_t = static_cast<int>(t);
+                    } else {
+                        db = b_cur;
+                        dt = static_cast<int>(t);
+                        dbuf = u & 1;
+                    }
+                    b_cur = -1;
+                }
+                if (db >= 0) {
+                    named_sync_softmax();
+                    if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(42, t);
+                    sm_drain<N, KOWN>(c, a, ss, bars, db, dt, dbuf);
+                    if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(43, t);
+                    if (ss.sm_fail) break;
+                }
+            }
+            if (ss.sm_fail) break;
+        }
     }
     named_sync_softmax();
-    if (b_cur >= 0 && !ss.sm_fail) sm_epilogue<N, KOWN>(c, a, ss, bars, l_part, b_cur, t_last);
+    if constexpr (kOBufs<N> == 1) {
+        if (b_cur >= 0 && !ss.sm_fail) sm_epilogue<N, KOWN>(c, a, ss, bars, l_part, b_cur, t_prev);
+    }
 }
 
 // N: query rows per CTA (multiple of 16, <= 80).  CL: CTAs per cluster (1 or 2).
@@ -547,7 +705,7 @@ __global__ void __maxnreg__(128)
 {
     constexpr uint16_t kMask = (1u << CL) - 1;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
-    __shared__ Bars bars;
+    __shared__ BarsT<N> bars;
     __shared__ Shared<N> ss;
     __shared__ int64_t red64[32];
 
@@ -586,6 +744,7 @@ __global__ void __maxnreg__(128)
             mbar_init(&bars.pv_done[i], 1);
         }
         mbar_init(&bars.o_free, kSoftmaxWarps);
+        if constexpr (kOBufs<N> == 2) mbar_init(o_free_bar(bars, 1), kSoftmaxWarps);
         mbar_init(&bars.drain_qk, 1);
         mbar_init(&bars.drain_pv, 1);
 #ifdef GBMLA_TRACE
@@ -599,8 +758,7 @@ __global__ void __maxnreg__(128)
         tc::fence_barrier_init();
     }
     if (warp == 1) {
-        constexpr uint32_t cols = (2 * N + 4 * N) <= 128 ? 128 : ((2 * N + 4 * N) <= 256 ? 256 : 512);
-        tc::tmem_alloc(smem_u32(&ss.tmem_base), cols);
+        tc::tmem_alloc(smem_u32(&ss.tmem_base), kTmemCols<N>);
         tc::tmem_relinquish();
     }
     tc::fence_before_sync();
@@ -628,8 +786,15 @@ __global__ void __maxnreg__(128)
     const int64_t t_begin = T ? part_begin(part, T, a.num_splits) : 0;
     const int64_t t_end = T ? part_begin(part + 1, T, a.num_splits) : 0;
     const int n_items = static_cast<int>(t_end - t_begin);
+#ifdef GBMLA_TRACE
+    if (tid == 0) {
+        const int64_t cta = static_cast<int64_t>(blockIdx.y) * gridDim.x + blockIdx.x;
+        GBMLA_TRACE_CTA(30, cta);
+        GBMLA_TRACE_CTA(32, (cta << 32) | (t_begin << 8) | n_items);
+    }
+#endif
     const uint32_t tmem = ss.tmem_base;
-    const uint32_t o_col0 = 2 * N;   // S^T buffers at columns [0, N) and [N, 2N)
+    const uint32_t o_col0 = 2 * N;   // S^T buffers at columns [0, N) and [N, 2N); O^T buffer i at 2N + 4N i
     auto any_abort = [&]() {
         return __any_sync(0xffffffffu, *reinterpret_cast<volatile int *>(&ss.abort) != 0);
     };
@@ -707,6 +872,7 @@ __global__ void __maxnreg__(128)
                         if (kind == kQuery) {
                             const int box = lane - 16;
                             if (box == 0) tc::mbar_arrive_expect_tx(fbar, nqc * N * 128);
+                            if (box == 0) GBMLA_TRACE_EVENT(40, w.b);
                             tc::tma_load_2d(dst, &map_q, 64 * box, w.b * a.rows + group * N, fbar);
                             do {
                                 w.next();
@@ -802,6 +968,7 @@ __global__ void __maxnreg__(128)
                     if (w.first()) {
                         ++seg;
                         if (!wait(&bars.q_full, seg & 1)) break;
+                        if (lane == 0) GBMLA_TRACE_EVENT(41, t);
                     }
                     const int sb = t & 1;
                     if (lane == 0) GBMLA_TRACE_EVENT(2, t);
@@ -832,14 +999,19 @@ __global__ void __maxnreg__(128)
                 const uint32_t id_pv = tc::idesc_bf16_f32(128, N, true, true);
                 const uint32_t ring_base = smem_u32(ring_b);
                 int seg = -1;
+                uint32_t o_cur = o_col0;
                 for (int t = 0; t < n_items && ok; ++t, w.next()) {
                     if (any_abort()) break;
                     if (!wait(&bars.p_full[t % kPBufs<N>], (t / kPBufs<N>) & 1)) break;
                     if (lane == 0) GBMLA_TRACE_EVENT(4, t);
                     bool first_pv = false;
                     if (w.first()) {
+                        // buffer seg % kOBufs: wait until the sequence that used it last has drained
                         ++seg;
-                        if (seg >= 1 && !wait(&bars.o_free, (seg - 1) & 1)) break;
+                        const int ob = seg % kOBufs<N>, use = seg / kOBufs<N>;
+                        if (use >= 1 && !wait(o_free_bar(bars, ob), (use - 1) & 1)) break;
+                        o_cur = o_col0 + static_cast<uint32_t>(ob * 4 * N);
+                        if (lane == 0) GBMLA_TRACE_EVENT(44, t);
                         first_pv = true;
                     }
                     // A sequence's last, partial tile of v rows: only the 16-token
@@ -868,7 +1040,7 @@ __global__ void __maxnreg__(128)
                         }
                         const uint32_t cb = ring_base + s0 * kChunkBytes;
                         const uint32_t pb = p_base + (t % kPBufs<N>) * (N / 16) * (kTile * 32);
-                        const uint32_t d_o = tmem + o_col0 + m * N;
+                        const uint32_t d_o = tmem + o_cur + m * N;
                         for (int kk = 0; kk < v16 / 16; ++kk)
                             tc::mma_bf16_elect(d_o, with_addr(dc, cb + kk * 16 * 128),
                                                with_addr(dp, pb + kk * 16 * 32), id_pv,
@@ -937,11 +1109,11 @@ __global__ void __maxnreg__(128)
 
     tc::fence_before_sync();
     __syncthreads();
+    if (tid == 0) GBMLA_TRACE_CTA(31, static_cast<int64_t>(blockIdx.y) * gridDim.x + blockIdx.x);
     if (CL > 1) tc::cluster_sync();  // no CTA leaves while a peer may still signal it
     if (warp == 1) {
         tc::fence_after_sync();
-        constexpr uint32_t cols = (2 * N + 4 * N) <= 128 ? 128 : ((2 * N + 4 * N) <= 256 ? 256 : 512);
-        tc::tmem_dealloc(tmem, cols);
+        tc::tmem_dealloc(tmem, kTmemCols<N>);
     }
 }
 
@@ -1004,7 +1176,7 @@ cudaError_t launch_cfg(const AttnArgs &a, int groups, cudaStream_t st)
     int dev = 0, optin = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-    const int static_bytes = static_cast<int>(sizeof(Bars) + sizeof(Shared<N>) + 32 * 8) + 128;
+    const int static_bytes = static_cast<int>(sizeof(BarsT<N>) + sizeof(Shared<N>) + 32 * 8) + 128;
     int slots = (optin - static_bytes - fixed - p_bytes) / kChunkBytes;
     if (slots > kMaxSlots) slots = kMaxSlots;
     if (const char *env = getenv("GBMLA_TC_MAX_SLOTS")) {  // testing aid: smaller rings
@@ -1117,5 +1289,10 @@ extern "C" int mla_debug_trace(unsigned long long *buf, unsigned cap)
     if (cudaMemcpyToSymbol(gbmla::g_trace_cap, &cap, sizeof cap) != cudaSuccess) return 1;
     if (cudaMemcpyToSymbol(gbmla::g_trace_count, &zero, sizeof zero) != cudaSuccess) return 1;
     return 0;
+}
+
+extern "C" int mla_debug_trace_cta(unsigned which)
+{
+    return cudaMemcpyToSymbol(gbmla::g_trace_which, &which, sizeof which) != cudaSuccess;
 }
 #endif
