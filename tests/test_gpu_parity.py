@@ -244,7 +244,10 @@ def test_tensor_core_kernel_shapes_and_rings(env, splits, monkeypatch):
     """Several sequences per CTA, tail tiles of one or two pages, and rings
     smaller than a tile's chunk count (the regime where a look-ahead barrier
     wait once cleared the next sequence's rows): every query-group size,
-    cluster mode and ring size matches the oracle."""
+    cluster mode and ring size matches the oracle.  With 32 and 48 rows the
+    kernel alternates two O^T buffers between sequences and drains each after
+    the next one's first tile; one split puts all five sequences in one CTA,
+    so both buffers are reused and every deferred drain runs."""
     for k, v in env.items():
         monkeypatch.setenv(k, v)
     shape = wl.SHAPES["llama1b_paged_b128_h32_r512_t128_8192"]
