@@ -238,10 +238,14 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
     // rows from its stage base: the rows past RT come from the next stages or
     // the B ring (inside the allocation), land in accumulator rows >= RT and
     // are never stored.
-    const int AS = (AF32 || PROJ) ? kABytes : p.a_stride;
-    unsigned char *sa = smem;                            // NS x A tile
+    // An fp32 A has no A stages of its own: each converter thread writes its
+    // bf16 row over the first half of its raw fp32 row, which it has read
+    // before (chunk j of the row is written after the step that read it), so
+    // a stage's bf16 tile is the first 16 KB of its raw stage.
+    const int AS = AF32 ? 0 : PROJ ? kABytes : p.a_stride;
+    unsigned char *sa = smem;                            // NS x A tile (bf16 A)
     unsigned char *sb = sa + NS * AS;                    // NS x B tile
-    unsigned char *sr = sb + NS * kBBytes;               // NS x raw fp32 A (AF32)
+    unsigned char *sr = sb + NS * kBBytes;               // NS x raw fp32 A, then its bf16 tile (AF32)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int R = p.rblk, RT = R * p.hpg;                // row blocks and rows per tile (<= 128)
     const int mt = blockIdx.x / ks, n0 = blockIdx.y * BN, g = blockIdx.z;
@@ -338,7 +342,7 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
                                              (!AF32 || mbar_wait(smem_u32(&bars.conv_done[s]), par, lim)));
             if (!ok) break;
             tc::fence_after_sync();
-            const uint32_t a_base = smem_u32(sa + s * AS), b_base = smem_u32(sb + s * kBBytes);
+            const uint32_t a_base = smem_u32(AF32 ? sr + s * kRawBytes : sa + s * AS), b_base = smem_u32(sb + s * kBBytes);
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk) {
                 const uint32_t b_addr = NMAJ ? b_base + kk * 16 * 128 : b_base + kk * 32;
@@ -361,7 +365,7 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_tc_kernel(const __grid_cons
                 }
                 const uint4 *src0 = reinterpret_cast<const uint4 *>(sr + s * kRawBytes + r * 128);
                 const uint4 *src1 = reinterpret_cast<const uint4 *>(sr + s * kRawBytes + 128 * 128 + r * 128);
-                uint4 *dst = reinterpret_cast<uint4 *>(sa + s * AS + r * 128);
+                uint4 *dst = reinterpret_cast<uint4 *>(sr + s * kRawBytes + r * 128);  // over src0, in place
 #pragma unroll
                 for (int j = 0; j < 8; ++j) {
                     // bf16 16-byte chunk j = fp32 chunks 2j, 2j + 1 (of box j / 4)
@@ -569,7 +573,7 @@ template <int BN, bool AF32>
 int ring_stages(int K, size_t *smem)
 {
     const int nk = (K + 63) / 64;
-    const size_t per_stage = 128 * 128 + BN * 128 + (AF32 ? 2 * 128 * 128 : 0);
+    const size_t per_stage = (AF32 ? 2 * 128 * 128 : 128 * 128) + BN * 128;  // fp32 A: raw stage, bf16 in place
     int ns = static_cast<int>((192 * 1024) / per_stage);
     if (ns > kStages) ns = kStages;
     if (ns > nk) ns = nk;
@@ -645,9 +649,16 @@ cudaError_t launch_tc(const GroupGemm &p, cudaStream_t st, const ProjEpi *rope =
         smem = 1024 + (ring > window ? ring : window);
     } else {
         q.stages = ring_stages<BN, AF32>((nk + ks - 1) / ks * 64, &smem);
+        const size_t per_stage = (AF32 ? 2 * 128 * 128 : 128 * 128) + BN * 128;
         if (ks > 1 && !wide_split && q.stages > 4) {
             q.stages = 4;
-            smem = 1024 + 4 * (128 * 128 + BN * 128 + (AF32 ? 2 * 128 * 128 : 0));
+            smem = 1024 + 4 * per_stage;
+        }
+        // an fp32-A grid just past one CTA per SM (W_UV of a large batch):
+        // two stages, so that two CTAs share an SM and the grid runs in one wave
+        if (AF32 && ks == 1 && tiles > 152 && tiles <= 2 * 152 && q.stages > 2) {
+            q.stages = 2;
+            smem = 1024 + 2 * per_stage;
         }
     }
     q.rblk = rblk;
