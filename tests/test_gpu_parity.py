@@ -256,3 +256,26 @@ def test_tensor_core_kernel_shapes_and_rings(env, splits, monkeypatch):
     ref = oracle_step(w)
     assert_close(step.o_lat.cpu().numpy(), ref["o_lat"], "o_lat")
     assert_close(step.lse.cpu().numpy(), ref["lse"], "lse")
+
+
+@pytest.mark.parametrize("name,groups", [("tiny_b1_h8_r128_t256", 1), ("qwen05b_b16_h14_r256_t2048", 1),
+                                         ("llama3b_long_b8_h24_r512_t16k_32k", 1),
+                                         ("llama1b_chunk5_b32_h32_r512_t4096", 2)])
+def test_automatic_split_count(name, groups):
+    """num_splits = 0 resolves by the rule mla_workspace_size documents: one
+    partition per SM (per pair of SMs for two query groups), capped by the
+    tile count T = batch ceil(max_kv_len / 128); when that leaves at most four
+    tiles per partition, the fewest partitions with the same most tiles."""
+    s = wl.SHAPES[name]
+    dims = abi.Dims(s.num_heads, s.num_kv_groups, s.d_nope, s.d_rope, s.d_v, s.rank, s.hidden, s.sm_scale,
+                    s.rope_style, s.rope_base)
+    max_kv = s.kv_hi
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    tiles = s.batch * -(-max_kv // abi.SPLIT_TILE)
+    want = max(1, min(sms // groups, tiles))
+    per = -(-tiles // want)
+    if per <= 4:
+        want = -(-tiles // per)
+    assert abi.workspace_size(dims, s.batch, s.q_len, max_kv)[2] == want
+    # a requested count is taken as given
+    assert abi.workspace_size(dims, s.batch, s.q_len, max_kv, 7)[2] == 7
