@@ -314,9 +314,12 @@ mla_status mla_e2e_loss(int32_t rows, int32_t hidden, const void *a_mla, const v
  *   The first call on a device looks up the array's device address with that
  *   device current (a host-side query); make that first call before any stream
  *   capture.  Every call uses the same array, so calls that overlap on the GPU
- *   (different streams, or different threads) race and must be serialised;
- *   each call writes every partial it later reads, so nothing has to start at
- *   zero and stale contents from an earlier call are never used. */
+ *   (different streams, or different threads) race and must be serialised.
+ *   Nothing in the array has to start at zero: each call writes the partial
+ *   of every (sequence, partition) pair that holds tiles before its combine
+ *   reads it.  The slots of empty partitions (fewer tiles than partitions)
+ *   may hold stale data from an earlier call; the combine loads them but
+ *   gives them zero weight, so they never reach an output. */
 mla_status mla_decode_attn_noalloc(const mla_dims *dims, const mla_cache *cache, int32_t batch, int32_t q_len,
                                    const int32_t *kv_len, int32_t max_kv_len, const void *q_abs, int32_t num_splits,
                                    float *o_lat, float *lse, void *stream);
@@ -332,6 +335,15 @@ mla_status mla_check_status(void *stream);
  * MLA_ERR_DEVICE_TIMEOUT.  Returns the launch status only; read the outcome
  * with mla_check_status(). */
 mla_status mla_selftest_wait_timeout(int64_t limit_ns, void *stream);
+
+/* Testing aid: re-read the GBMLA_* environment variables that choose the
+ * attention kernel's tiling (they are otherwise read once per process, at the
+ * first call that needs them): GBMLA_ATTN_KERNEL=simt (CUDA-core attention),
+ * GBMLA_TC_MAX_N (query rows per tensor-core CTA, 16..80), GBMLA_TC_MAX_SLOTS
+ * and GBMLA_TC_PV_SLOTS (ring slots).  Results are the same under every
+ * setting, up to the floating-point order of the split partials.  Not
+ * thread-safe against concurrent launches; the paper has no counterpart. */
+void mla_reload_tuning(void);
 
 /* Text of the CUDA error behind the last MLA_ERR_CUDA returned to the calling
  * thread ("" if none).  The library's own; it has no counterpart in the

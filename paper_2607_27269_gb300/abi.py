@@ -23,7 +23,7 @@ EXPORTS = ("mla_workspace_size", "mla_cache_append", "mla_project_append", "mla_
            "mla_gqa_append", "mla_gqa_workspace_size", "mla_gqa_decode_attn", "mla_gqa_project", "mla_gqa_out_proj",
            "mla_e2e_loss", "mla_absorb_q", "mla_decode_attn", "mla_combine",
            "mla_out_proj", "mla_check_status", "mla_selftest_wait_timeout", "mla_decode_attn_noalloc",
-           "mla_status_str", "mla_last_error")
+           "mla_reload_tuning", "mla_status_str", "mla_last_error")
 
 
 class MlaError(RuntimeError):
@@ -65,7 +65,7 @@ def lib(auto_build: bool = True):
     global _lib
     with _lock:
         if _lib is None:
-            # GBMLA_LIBRARY selects another build of the library (e.g. the trace build)
+            # GBMLA_LIBRARY selects another build of the library
             path = os.environ.get("GBMLA_LIBRARY") or (_build.build() if auto_build else _build.LIB)
             if not os.path.exists(path):
                 raise RuntimeError(f"libgbmla.so is missing at {path}; run paper_2607_27269_gb300.build.build()")
@@ -94,10 +94,17 @@ def lib(auto_build: bool = True):
             L.mla_decode_attn_noalloc.argtypes = [P(MlaDims), P(MlaCache), i32, i32, vp, i32, vp, i32, vp, vp, vp]
             L.mla_last_error.restype = ctypes.c_char_p
             L.mla_last_error.argtypes = []
-            for name in EXPORTS[:-2]:
+            for name in EXPORTS[:-3]:
                 getattr(L, name).restype = ctypes.c_int
+            L.mla_reload_tuning.restype = None
+            L.mla_reload_tuning.argtypes = []
             _lib = L
         return _lib
+
+
+def reload_tuning() -> None:
+    """Re-read the GBMLA_* testing variables (mla_reload_tuning)."""
+    lib().mla_reload_tuning()
 
 
 def status_name(code: int) -> str:

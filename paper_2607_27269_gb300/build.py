@@ -18,7 +18,6 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(os.path.dirname(PKG), "include")
 BUILD_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libgbmla.so")
-LIB_TRACE = os.path.join(PKG, "libgbmla_trace.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 SOURCES = ["accept.cu", "api.cu", "append.cu", "absorb.cu", "e2e.cu", "attn_simt.cu", "attn_tc.cu", "combine.cu", "gemm.cu", "gqa.cu", "out_proj.cu"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
@@ -46,17 +45,15 @@ def is_stale(lib_path: str = LIB) -> bool:
     return any(os.path.getmtime(f) > t for f in _inputs())
 
 
-def build(force: bool = False, verbose: bool = False, extra_flags=None, trace: bool = False) -> str:
-    """Compile every .cu of csrc/ and link libgbmla.so; returns its path.
-    trace=True builds libgbmla_trace.so instead, with the per-CTA event trace
-    of the attention kernel compiled in (a development aid)."""
-    lib_path = LIB_TRACE if trace else LIB
-    build_dir = BUILD_DIR + ("_trace" if trace else "")
+def build(force: bool = False, verbose: bool = False, extra_flags=None) -> str:
+    """Compile every .cu of csrc/ and link libgbmla.so; returns its path."""
+    lib_path = LIB
+    build_dir = BUILD_DIR
     if not force and not is_stale(lib_path):
         return lib_path
     os.makedirs(build_dir, exist_ok=True)
     nvcc = _nvcc()
-    flags = NVCC_FLAGS + list(extra_flags or []) + (["-DGBMLA_TRACE"] if trace else [])
+    flags = NVCC_FLAGS + list(extra_flags or [])
 
     def compile_one(src):
         obj = os.path.join(build_dir, src.replace(".cu", ".o"))
@@ -80,4 +77,4 @@ def build(force: bool = False, verbose: bool = False, extra_flags=None, trace: b
 
 
 if __name__ == "__main__":
-    print(build(force="--force" in sys.argv, verbose=True, trace="--trace" in sys.argv))
+    print(build(force="--force" in sys.argv, verbose=True))

@@ -86,12 +86,11 @@ mla_status check_cache(const mla_dims *d, const mla_cache *c, CacheView *v)
 }
 
 // The tensor-core kernel serves every shape with rank % 128 == 0; the
-// CUDA-core kernel serves the rest.  GBMLA_ATTN_KERNEL=simt forces the
+// CUDA-core kernel serves the rest.  The attn_simt testing aid forces the
 // CUDA-core kernel (used by tests that compare the two).
 bool use_tc_kernel(const mla_dims *d)
 {
-    const char *env = getenv("GBMLA_ATTN_KERNEL");
-    if (env && strcmp(env, "simt") == 0) return false;
+    if (tuning().attn_simt) return false;
     return d->rank % 128 == 0;
 }
 
@@ -125,6 +124,27 @@ int resolve_splits(const mla_dims *d, int batch, int q_len, int max_kv_len, int 
 }
 
 thread_local cudaError_t g_last_cuda_error = cudaSuccess;
+
+Tuning g_tuning;
+std::once_flag g_tuning_once;
+
+int env_int(const char *name)
+{
+    const char *v = getenv(name);
+    return v ? atoi(v) : 0;
+}
+
+void read_tuning()
+{
+    Tuning t;
+    const char *k = getenv("GBMLA_ATTN_KERNEL");
+    t.attn_simt = (k && strcmp(k, "simt") == 0) ? 1 : 0;
+    t.tc_max_rows = env_int("GBMLA_TC_MAX_N");
+    t.tc_max_slots = env_int("GBMLA_TC_MAX_SLOTS");
+    t.tc_pv_slots = env_int("GBMLA_TC_PV_SLOTS");
+    std::lock_guard<std::mutex> lock(g_mutex);
+    g_tuning = t;
+}
 
 // Scratch of mla_decode_attn_noalloc: the split partials live here instead of
 // in caller buffers.  32 MiB, reserved on every device that loads the library
@@ -173,6 +193,18 @@ __global__ void selftest_wait_kernel(uint64_t limit_ns, unsigned *status)
 }
 
 }  // namespace
+
+const Tuning &tuning()
+{
+    std::call_once(g_tuning_once, read_tuning);
+    return g_tuning;
+}
+
+void reload_tuning()
+{
+    std::call_once(g_tuning_once, read_tuning);
+    read_tuning();
+}
 
 cudaError_t launch_selftest_wait(int64_t limit_ns, unsigned *status, cudaStream_t st)
 {
@@ -630,6 +662,8 @@ const char *mla_last_error(void)
 {
     return g_last_cuda_error == cudaSuccess ? "" : cudaGetErrorString(g_last_cuda_error);
 }
+
+void mla_reload_tuning(void) { reload_tuning(); }
 
 mla_status mla_selftest_wait_timeout(int64_t limit_ns, void *stream)
 {

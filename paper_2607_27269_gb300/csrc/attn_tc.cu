@@ -10,9 +10,9 @@
 // rings of 64-column chunks: the QK ring (positional keys, then the latent
 // chunks of each tile) feeds the score products, the PV ring (the latent
 // chunks again, from L2) the value products, so that the softmax of tile t
-// overlaps QK(t+1) and PV(t-1).  With two query groups (160 query rows) the
-// two CTAs form a cluster and every cache box is multicast to both, so each
-// byte leaves L2 once per pass.  A sequence's last, partial tile issues only
+// overlaps QK(t+1) and PV(t-1).  More than 80 query rows run as several
+// independent CTAs per partition, each loading the cache boxes itself (the
+// later ones hit in L2).  A sequence's last, partial tile issues only
 // the value products of its 16-token steps that hold cached rows; the PV warp
 // clears the rows past the end inside the last such step itself.
 //
@@ -57,42 +57,6 @@ template <int N>
 constexpr uint32_t kTmemCols = (2 * N + kOBufs<N> * 4 * N) <= 128 ? 128u
                                : (2 * N + kOBufs<N> * 4 * N) <= 256 ? 256u : 512u;
 
-// Optional event trace (compiled only with -DGBMLA_TRACE): (globaltimer ns,
-// event code, argument) triples in a caller buffer of 2 cap entries (two
-// 64-bit words each), set by mla_debug_trace(buf, cap): entries 0 .. cap - 1
-// hold the role timeline of one CTA (mla_debug_trace_cta picks it, default
-// 0), entries cap .. 2 cap - 1 every CTA's start, end and tile range.
-#ifdef GBMLA_TRACE
-__device__ unsigned long long *g_trace_buf;
-__device__ unsigned g_trace_count;
-__device__ unsigned g_trace_cap;
-__device__ unsigned g_trace_which;  // the CTA (y * gridDim.x + x) whose roles are traced
-__shared__ unsigned s_trace_count;  // events of this CTA (a shared-memory atomic keeps the probe cheap)
-__device__ __forceinline__ void trace_event(int code, int64_t arg)
-{
-    if (blockIdx.y * gridDim.x + blockIdx.x != g_trace_which || g_trace_buf == nullptr) return;
-    const unsigned i = atomicAdd(&s_trace_count, 1u);
-    if (i >= g_trace_cap) return;
-    g_trace_buf[2 * i] = global_ns();
-    g_trace_buf[2 * i + 1] = (static_cast<unsigned long long>(code) << 48) | (static_cast<unsigned long long>(arg) & 0xffffffffffffull);
-}
-// Every CTA: (time, code, argument) of its start, end and tile range, in
-// entries cap .. 2 cap - 1 of the same buffer.
-__device__ __forceinline__ void trace_cta(int code, int64_t arg)
-{
-    if (g_trace_buf == nullptr) return;
-    const unsigned i = atomicAdd(&g_trace_count, 1u);
-    if (i >= g_trace_cap) return;
-    g_trace_buf[2 * (g_trace_cap + i)] = global_ns();
-    g_trace_buf[2 * (g_trace_cap + i) + 1] =
-        (static_cast<unsigned long long>(code) << 48) | (static_cast<unsigned long long>(arg) & 0xffffffffffffull);
-}
-#define GBMLA_TRACE_EVENT(code, arg) trace_event((code), (arg))
-#define GBMLA_TRACE_CTA(code, arg) trace_cta((code), (arg))
-#else
-#define GBMLA_TRACE_EVENT(code, arg) ((void)0)
-#define GBMLA_TRACE_CTA(code, arg) ((void)0)
-#endif
 
 struct TcArgs {
     int batch, q_len, heads, rank, d_rope, rows, num_splits, max_kv;
@@ -311,24 +275,10 @@ struct SmCtx {
 
 // The whole warp waits; a failure marks sm_fail, which the softmax
 // warps read only after their next named barrier, so they all leave together.
-#ifdef GBMLA_TRACE
-__shared__ unsigned long long s_sm_wait_cyc;
-#endif
 template <int N>
 __device__ __forceinline__ void sm_wait(const SmCtx &c, const TcArgs &a, Shared<N> &ss, uint64_t *bar,
                                         uint32_t parity)
 {
-#ifdef GBMLA_TRACE
-    const long long w0 = clock64();
-    struct Acc {
-        long long t0;
-        int lane;
-        __device__ ~Acc()
-        {
-            if (lane == 0) atomicAdd(&s_sm_wait_cyc, static_cast<unsigned long long>(clock64() - t0));
-        }
-    } acc{w0, c.lane};
-#endif
     if (!__all_sync(0xffffffffu, mbar_wait(smem_u32(bar), parity, c.lim_ns)) && c.lane == 0) {
         record_status(a.status, kStatusTimeout);
         atomicOr(&ss.sm_fail, 1);
@@ -511,7 +461,6 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
         const int kv = a.kv_len[b];
         const int sb = static_cast<int>(t & 1);
         sm_wait<N>(c, a, ss, &bars.s_full[sb], static_cast<uint32_t>((t >> 1) & 1));
-        if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(6, t);
         named_sync_softmax();
         if (ss.sm_fail) break;
         tc::fence_after_sync();
@@ -589,11 +538,9 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
         // completed; O^T is rescaled (rarely: only when a base moves) once
         // PV(t-1) has completed.  Each wait is on the next phase of its barrier.
         constexpr int NP = kPBufs<N>;
-        if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(7, t);
         if (t >= NP) sm_wait<N>(c, a, ss, &bars.pv_done[t % NP], static_cast<uint32_t>(((t - NP) / NP) & 1));
         if (ss.any_rescale)  // never on a sequence's first tile
             sm_wait<N>(c, a, ss, &bars.pv_done[(t - 1) % NP], static_cast<uint32_t>(((t - 1) / NP) & 1));
-        if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(8, t);
         named_sync_softmax();
         if (ss.sm_fail) break;
         tc::fence_after_sync();
@@ -652,7 +599,6 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
         tc::fence_before_sync();
         __syncwarp();
         if (c.lane == 0) tc::mbar_arrive(smem_u32(&bars.p_full[t % kPBufs<N>]));
-        if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(9, t);
         if constexpr (kOBufs<N> == 2) {
             // Due now, in this order: the previous sequence's drain (deferred
             // until this first P was out, so that it overlaps this tile's value
@@ -682,9 +628,7 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
                 }
                 if (db >= 0) {
                     named_sync_softmax();
-                    if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(42, t);
                     sm_drain<N, KOWN>(c, a, ss, bars, db, dt, dbuf);
-                    if (c.tid == kSoftmaxBase) GBMLA_TRACE_EVENT(43, t);
                     if (ss.sm_fail) break;
                 }
             }
@@ -697,13 +641,12 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
     }
 }
 
-// N: query rows per CTA (multiple of 16, <= 80).  CL: CTAs per cluster (1 or 2).
-template <int N, int CL>
+// N: query rows per CTA (multiple of 16, <= 80).
+template <int N>
 __global__ void __maxnreg__(128)
     attn_tc_kernel(const __grid_constant__ TcArgs a, const __grid_constant__ CUtensorMap map_c,
                    const __grid_constant__ CUtensorMap map_r, const __grid_constant__ CUtensorMap map_q)
 {
-    constexpr uint16_t kMask = (1u << CL) - 1;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     __shared__ BarsT<N> bars;
     __shared__ Shared<N> ss;
@@ -723,15 +666,14 @@ __global__ void __maxnreg__(128)
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int group = blockIdx.x, part = blockIdx.y;
-    const uint32_t rank_in_cluster = CL > 1 ? tc::cluster_ctarank() : 0;
     const uint64_t lim_ns = a.wait_ns;
 
     if (tid == 0) {
         for (int i = 0; i < kMaxSlots; ++i) {
             mbar_init(&bars.qk_full[i], 1);
-            mbar_init(&bars.qk_empty[i], CL);
+            mbar_init(&bars.qk_empty[i], 1);
             mbar_init(&bars.pv_full[i], 1);
-            mbar_init(&bars.pv_empty[i], CL);
+            mbar_init(&bars.pv_empty[i], 1);
         }
         mbar_init(&bars.q_full, 1);
         mbar_init(&bars.q_free, 1);
@@ -747,10 +689,6 @@ __global__ void __maxnreg__(128)
         if constexpr (kOBufs<N> == 2) mbar_init(o_free_bar(bars, 1), kSoftmaxWarps);
         mbar_init(&bars.drain_qk, 1);
         mbar_init(&bars.drain_pv, 1);
-#ifdef GBMLA_TRACE
-        s_trace_count = 0;
-        s_sm_wait_cyc = 0;
-#endif
         ss.need_max = 0;
         ss.any_rescale = 0;
         ss.abort = 0;
@@ -763,7 +701,6 @@ __global__ void __maxnreg__(128)
     }
     tc::fence_before_sync();
     __syncthreads();
-    if (CL > 1) tc::cluster_sync();  // peers may multicast into this CTA only after its barriers exist
     tc::fence_after_sync();
     // The queries come from the previous launch; the cache does not: every
     // kernel of this library that writes the cache (append, projection) lets
@@ -786,13 +723,6 @@ __global__ void __maxnreg__(128)
     const int64_t t_begin = T ? part_begin(part, T, a.num_splits) : 0;
     const int64_t t_end = T ? part_begin(part + 1, T, a.num_splits) : 0;
     const int n_items = static_cast<int>(t_end - t_begin);
-#ifdef GBMLA_TRACE
-    if (tid == 0) {
-        const int64_t cta = static_cast<int64_t>(blockIdx.y) * gridDim.x + blockIdx.x;
-        GBMLA_TRACE_CTA(30, cta);
-        GBMLA_TRACE_CTA(32, (cta << 32) | (t_begin << 8) | n_items);
-    }
-#endif
     const uint32_t tmem = ss.tmem_base;
     const uint32_t o_col0 = 2 * N;   // S^T buffers at columns [0, N) and [N, 2N); O^T buffer i at 2N + 4N i
     auto any_abort = [&]() {
@@ -872,7 +802,6 @@ __global__ void __maxnreg__(128)
                         if (kind == kQuery) {
                             const int box = lane - 16;
                             if (box == 0) tc::mbar_arrive_expect_tx(fbar, nqc * N * 128);
-                            if (box == 0) GBMLA_TRACE_EVENT(40, w.b);
                             tc::tma_load_2d(dst, &map_q, 64 * box, w.b * a.rows + group * N, fbar);
                             do {
                                 w.next();
@@ -886,21 +815,13 @@ __global__ void __maxnreg__(128)
                             const bool keys = kind == kQK && i == 0;
                             const CUtensorMap *map = keys ? &map_r : &map_c;
                             const int col = keys ? 0 : 64 * (kind == kQK ? i - 1 : i);
-                            if (lane == 0 && warp == 0) GBMLA_TRACE_EVENT(1, c);
                             tc::mbar_arrive_expect_tx(fbar, L.bytes);
-                            if (c % CL == rank_in_cluster) {
-                                // the QK pass keeps latent lines in L2 for the PV pass, which reads
-                                // them a last time; the positional keys are read once
-                                const uint64_t pol = (kind == kQK && !keys) ? pol_keep : pol_drop;
-                                for (int h = 0; h < L.nh; ++h) {
-                                    if (CL > 1)
-                                        tc::tma_load_3d_multicast_hint(dst + h * kHalf * 128, map, col, L.tok0[h],
-                                                                       L.blk[h], fbar, kMask, pol);
-                                    else
-                                        tc::tma_load_3d_hint(dst + h * kHalf * 128, map, col, L.tok0[h], L.blk[h],
-                                                             fbar, pol);
-                                }
-                            }
+                            // the QK pass keeps latent lines in L2 for the PV pass, which reads
+                            // them a last time; the positional keys are read once
+                            const uint64_t pol = (kind == kQK && !keys) ? pol_keep : pol_drop;
+                            for (int h = 0; h < L.nh; ++h)
+                                tc::tma_load_3d_hint(dst + h * kHalf * 128, map, col, L.tok0[h], L.blk[h], fbar,
+                                                     pol);
                             c += ring_len;
                             has = c < total;
                         }
@@ -938,27 +859,12 @@ __global__ void __maxnreg__(128)
             w.init(a.kv_len, a.batch, a.q_len, a.max_kv, t_begin, t_end);
             RingPos rp{0, 0};
             bool ok = true;
-#ifdef GBMLA_TRACE
-            long long wait_cyc = 0;
-            const long long loop_t0 = clock64();
-#endif
             auto wait = [&](uint64_t *bar, uint32_t parity) {
-#ifdef GBMLA_TRACE
-                const long long w0 = clock64();
-#endif
                 if (ok) ok = __all_sync(0xffffffffu, mbar_wait(smem_u32(bar), parity, lim_ns));
-#ifdef GBMLA_TRACE
-                wait_cyc += clock64() - w0;
-#endif
                 return ok;
             };
-            // a consumed slot is handed back to every CTA of the cluster
-            auto release = [&](uint64_t *bar) {
-                if (CL > 1)
-                    tc::commit_multicast_elect(smem_u32(bar), kMask);
-                else
-                    tc::commit_elect(smem_u32(bar));
-            };
+            // a consumed slot is handed back to its producer lane
+            auto release = [&](uint64_t *bar) { tc::commit_elect(smem_u32(bar)); };
             if (is_qk) {
                 const uint32_t id_qk = tc::idesc_bf16_f32(128, N, false, false);
                 const uint32_t ring_base = smem_u32(ring_a);
@@ -968,17 +874,11 @@ __global__ void __maxnreg__(128)
                     if (w.first()) {
                         ++seg;
                         if (!wait(&bars.q_full, seg & 1)) break;
-                        if (lane == 0) GBMLA_TRACE_EVENT(41, t);
                     }
                     const int sb = t & 1;
-                    if (lane == 0) GBMLA_TRACE_EVENT(2, t);
                     if (t >= 2 && !wait(&bars.s_free[sb], ((t >> 1) - 1) & 1)) break;
                     const uint32_t d_s = tmem + sb * N;
                     for (int i = 0; i < nqc && ok; ++i) {
-#ifdef GBMLA_TRACE
-                        if (lane == 0 && !mbar_test(smem_u32(&bars.qk_full[rp.slot]), rp.round & 1))
-                            GBMLA_TRACE_EVENT(12, static_cast<int64_t>(rp.round) * CA + rp.slot);
-#endif
                         if (!wait(&bars.qk_full[rp.slot], rp.round & 1)) break;
                         tc::fence_after_sync();
                         const uint32_t cb = ring_base + rp.slot * kChunkBytes;
@@ -992,7 +892,6 @@ __global__ void __maxnreg__(128)
                     }
                     if (!ok) break;
                     tc::commit_elect(smem_u32(&bars.s_full[sb]));
-                    if (lane == 0) GBMLA_TRACE_EVENT(3, t);
                     if (w.last()) tc::commit_elect(smem_u32(&bars.q_free));
                 }
             } else {
@@ -1003,7 +902,6 @@ __global__ void __maxnreg__(128)
                 for (int t = 0; t < n_items && ok; ++t, w.next()) {
                     if (any_abort()) break;
                     if (!wait(&bars.p_full[t % kPBufs<N>], (t / kPBufs<N>) & 1)) break;
-                    if (lane == 0) GBMLA_TRACE_EVENT(4, t);
                     bool first_pv = false;
                     if (w.first()) {
                         // buffer seg % kOBufs: wait until the sequence that used it last has drained
@@ -1011,7 +909,6 @@ __global__ void __maxnreg__(128)
                         const int ob = seg % kOBufs<N>, use = seg / kOBufs<N>;
                         if (use >= 1 && !wait(o_free_bar(bars, ob), (use - 1) & 1)) break;
                         o_cur = o_col0 + static_cast<uint32_t>(ob * 4 * N);
-                        if (lane == 0) GBMLA_TRACE_EVENT(44, t);
                         first_pv = true;
                     }
                     // A sequence's last, partial tile of v rows: only the 16-token
@@ -1052,19 +949,12 @@ __global__ void __maxnreg__(128)
                     }
                     if (!ok) break;
                     tc::commit_elect(smem_u32(&bars.pv_done[t % kPBufs<N>]));
-                    if (lane == 0) GBMLA_TRACE_EVENT(5, t);
                 }
             }
             if (!ok && lane == 0) {
                 record_status(a.status, kStatusTimeout);
                 ss.abort = 1;
             }
-#ifdef GBMLA_TRACE
-            if (lane == 0) {
-                GBMLA_TRACE_EVENT(is_qk ? 20 : 21, wait_cyc);
-                GBMLA_TRACE_EVENT(is_qk ? 22 : 23, clock64() - loop_t0);
-            }
-#endif
             // drain: every MMA this warp issued has completed before TMEM is freed
             tc::commit_elect(smem_u32(drain));
             if (!__all_sync(0xffffffffu, mbar_wait(smem_u32(drain), 0, lim_ns)) && lane == 0)
@@ -1094,23 +984,11 @@ __global__ void __maxnreg__(128)
         c.lim_ns = lim_ns;
         c.t_begin = t_begin;
         c.t_end = t_end;
-#ifdef GBMLA_TRACE
-        const long long sm_t0 = clock64();
-#endif
         softmax_role<N>(c, a, ss, bars);
-#ifdef GBMLA_TRACE
-        named_sync_softmax();
-        if (tid == kSoftmaxBase) {
-            GBMLA_TRACE_EVENT(24, static_cast<int64_t>(s_sm_wait_cyc / kSoftmaxWarps));
-            GBMLA_TRACE_EVENT(25, clock64() - sm_t0);
-        }
-#endif
     }
 
     tc::fence_before_sync();
     __syncthreads();
-    if (tid == 0) GBMLA_TRACE_CTA(31, static_cast<int64_t>(blockIdx.y) * gridDim.x + blockIdx.x);
-    if (CL > 1) tc::cluster_sync();  // no CTA leaves while a peer may still signal it
     if (warp == 1) {
         tc::fence_after_sync();
         tc::tmem_dealloc(tmem, kTmemCols<N>);
@@ -1145,7 +1023,7 @@ cudaError_t encode_cache_map(CUtensorMap *m, const void *base, int cols, int64_t
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-template <int N, int CL>
+template <int N>
 cudaError_t launch_cfg(const AttnArgs &a, int groups, cudaStream_t st)
 {
     cudaError_t e = get_encoder();
@@ -1179,20 +1057,14 @@ cudaError_t launch_cfg(const AttnArgs &a, int groups, cudaStream_t st)
     const int static_bytes = static_cast<int>(sizeof(BarsT<N>) + sizeof(Shared<N>) + 32 * 8) + 128;
     int slots = (optin - static_bytes - fixed - p_bytes) / kChunkBytes;
     if (slots > kMaxSlots) slots = kMaxSlots;
-    if (const char *env = getenv("GBMLA_TC_MAX_SLOTS")) {  // testing aid: smaller rings
-        const int cap = atoi(env);
-        if (cap >= 4 && cap < slots) slots = cap;
-    }
+    if (const int cap = tuning().tc_max_slots; cap >= 4 && cap < slots) slots = cap;  // testing aid: smaller rings
     if (slots < 4) return cudaErrorInvalidConfiguration;
     // the PV ring (refilled from L2) gets two or four slots, the QK ring the rest
     int pv_slots = slots >= 6 ? 4 : 2;
-    if (const char *env = getenv("GBMLA_TC_PV_SLOTS")) {  // testing aid
-        const int v = atoi(env) & ~1;
-        if (v >= 2 && v <= slots - 2) pv_slots = v;
-    }
+    if (const int v = tuning().tc_pv_slots & ~1; v >= 2 && v <= slots - 2) pv_slots = v;  // testing aid
     const int qk_slots = slots - pv_slots;
     const size_t smem = static_cast<size_t>(fixed) + static_cast<size_t>(slots) * kChunkBytes + p_bytes;
-    if ((e = cudaFuncSetAttribute(attn_tc_kernel<N, CL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if ((e = cudaFuncSetAttribute(attn_tc_kernel<N>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   static_cast<int>(smem))) != cudaSuccess)
         return e;
     TcArgs t;
@@ -1216,83 +1088,37 @@ cudaError_t launch_cfg(const AttnArgs &a, int groups, cudaStream_t st)
     t.lse_part = a.lse_part;
     t.status = a.status;
     t.wait_ns = kWaitLimitNs;
-    return launch_dependent(attn_tc_kernel<N, CL>, dim3(groups, a.num_splits, 1), dim3(kThreads), smem, st, CL, t,
-                            mc, mr, mq);
+    return launch_dependent(attn_tc_kernel<N>, dim3(groups, a.num_splits, 1), dim3(kThreads), smem, st, 1, t, mc,
+                            mr, mq);
 }
 
 }  // namespace
 
 TcShape attn_tc_shape(int rows)
 {
-    // Testing aids, read at every call: GBMLA_TC_MAX_N caps the query rows per
-    // CTA (16..80), GBMLA_TC_NO_CLUSTER=1 runs two query groups as separate
-    // CTAs (each loading the cache itself) instead of a multicast cluster.
-    int max_n = 80;
-    if (const char *e = getenv("GBMLA_TC_MAX_N")) max_n = atoi(e);
+    // Testing aid: the tuning knob tc_max_rows caps the query rows per CTA (16..80).
+    int max_n = tuning().tc_max_rows > 0 ? tuning().tc_max_rows : 80;
     if (max_n < 16) max_n = 16;
     if (max_n > 80) max_n = 80;
     max_n -= max_n % 16;
-    const bool no_cluster = getenv("GBMLA_TC_NO_CLUSTER") != nullptr;
     TcShape s;
-    if (max_n < 80) {
-        s.groups = (rows + max_n - 1) / max_n;
-        s.n = (((rows + s.groups - 1) / s.groups + 15) / 16) * 16;
-        s.cluster = 1;
-        return s;
-    }
-    if (rows <= 80) {
-        s.n = ((rows + 15) / 16) * 16;
-        s.groups = 1;
-        s.cluster = 1;
-    } else if (rows <= 160) {
-        s.n = (((rows + 1) / 2 + 15) / 16) * 16;
-        s.groups = 2;
-        s.cluster = no_cluster ? 1 : 2;
-    } else {
-        s.n = 80;
-        s.groups = (rows + 79) / 80;
-        s.cluster = 1;
-    }
+    s.groups = (rows + max_n - 1) / max_n;
+    s.n = (((rows + s.groups - 1) / s.groups + 15) / 16) * 16;
     return s;
 }
 
 cudaError_t launch_attn_tc(const AttnArgs &a, cudaStream_t st)
 {
     const TcShape s = attn_tc_shape(a.q_len * a.num_heads);
-    if (s.cluster == 2) {
-        switch (s.n) {
-        case 48: return launch_cfg<48, 2>(a, s.groups, st);
-        case 64: return launch_cfg<64, 2>(a, s.groups, st);
-        case 80: return launch_cfg<80, 2>(a, s.groups, st);
-        default: return cudaErrorInvalidConfiguration;
-        }
-    }
     switch (s.n) {
-    case 16: return launch_cfg<16, 1>(a, s.groups, st);
-    case 32: return launch_cfg<32, 1>(a, s.groups, st);
-    case 48: return launch_cfg<48, 1>(a, s.groups, st);
-    case 64: return launch_cfg<64, 1>(a, s.groups, st);
-    case 80: return launch_cfg<80, 1>(a, s.groups, st);
+    case 16: return launch_cfg<16>(a, s.groups, st);
+    case 32: return launch_cfg<32>(a, s.groups, st);
+    case 48: return launch_cfg<48>(a, s.groups, st);
+    case 64: return launch_cfg<64>(a, s.groups, st);
+    case 80: return launch_cfg<80>(a, s.groups, st);
     default: return cudaErrorInvalidConfiguration;
     }
 }
 
 }  // namespace gbmla
 
-#ifdef GBMLA_TRACE
-// Trace builds only: record the first CTA's events into `buf` (2 x 64-bit
-// words per event, at most `cap` events).  Returns the CUDA status.
-extern "C" int mla_debug_trace(unsigned long long *buf, unsigned cap)
-{
-    const unsigned zero = 0;
-    if (cudaMemcpyToSymbol(gbmla::g_trace_buf, &buf, sizeof buf) != cudaSuccess) return 1;
-    if (cudaMemcpyToSymbol(gbmla::g_trace_cap, &cap, sizeof cap) != cudaSuccess) return 1;
-    if (cudaMemcpyToSymbol(gbmla::g_trace_count, &zero, sizeof zero) != cudaSuccess) return 1;
-    return 0;
-}
-
-extern "C" int mla_debug_trace_cta(unsigned which)
-{
-    return cudaMemcpyToSymbol(gbmla::g_trace_which, &which, sizeof which) != cudaSuccess;
-}
-#endif

@@ -46,11 +46,21 @@ cudaError_t launch_absorb(const mla_dims &d, int batch, int q_len, const void *q
 constexpr int kSimtRows = 16;
 cudaError_t launch_attn_simt(const AttnArgs &a, cudaStream_t st);
 
+// Testing aids, read from the environment once per process (and again by
+// mla_reload_tuning): GBMLA_ATTN_KERNEL=simt (attn_simt = 1) forces the
+// CUDA-core attention; GBMLA_TC_MAX_N caps the query rows per tensor-core CTA;
+// GBMLA_TC_MAX_SLOTS caps its ring slots and GBMLA_TC_PV_SLOTS sets the share
+// of the value-product ring.  0 means "not set".  They change tiling only.
+struct Tuning {
+    int attn_simt, tc_max_rows, tc_max_slots, tc_pv_slots;
+};
+const Tuning &tuning();
+void reload_tuning();
+
 // Tensor-core attention core (tcgen05 + TMA).  For q_len * num_heads query
-// rows it runs `groups` CTAs of `n` rows per partition; with cluster == 2 the
-// two groups share every cache load through multicast.
+// rows it runs `groups` independent CTAs of `n` rows per partition.
 struct TcShape {
-    int n, groups, cluster;
+    int n, groups;
 };
 TcShape attn_tc_shape(int rows);
 cudaError_t launch_attn_tc(const AttnArgs &a, cudaStream_t st);

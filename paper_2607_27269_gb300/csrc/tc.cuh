@@ -100,16 +100,6 @@ __device__ __forceinline__ void commit_elect(uint32_t mbar)
         : "memory");
 }
 
-__device__ __forceinline__ void commit_multicast_elect(uint32_t mbar, uint16_t cta_mask)
-{
-    asm volatile(
-        "{\n .reg .pred e;\n elect.sync _|e, 0xffffffff;\n"
-        " @e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;\n}\n" ::"r"(
-            mbar),
-        "h"(cta_mask)
-        : "memory");
-}
-
 __device__ __forceinline__ void mbar_arrive_elect(uint32_t mbar)
 {
     asm volatile(
@@ -223,47 +213,6 @@ __device__ __forceinline__ void tma_load_3d_hint(uint32_t dst, const CUtensorMap
         "%3, %4}], [%5], %6;" ::"r"(dst),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(mbar), "l"(policy)
         : "memory");
-}
-
-__device__ __forceinline__ void tma_load_3d_multicast_hint(uint32_t dst, const CUtensorMap *map, int32_t c0,
-                                                           int32_t c1, int32_t c2, uint32_t mbar, uint16_t cta_mask,
-                                                           uint64_t policy)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster.L2::"
-        "cache_hint [%0], [%1, {%2, %3, %4}], [%5], %6, %7;" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(mbar), "h"(cta_mask), "l"(policy)
-        : "memory");
-}
-
-// Multicast variant: the box lands at the same shared-memory offset, and
-// signals the same-offset mbarrier, in every CTA of the cluster whose bit is
-// set in cta_mask.
-__device__ __forceinline__ void tma_load_3d_multicast(uint32_t dst, const CUtensorMap *map, int32_t c0, int32_t c1,
-                                                      int32_t c2, uint32_t mbar, uint16_t cta_mask)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster [%0], "
-        "[%1, {%2, %3, %4}], [%5], %6;" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(mbar), "h"(cta_mask)
-        : "memory");
-}
-
-// Arrive once on the same-offset mbarrier of every CTA in cta_mask when the
-// MMAs this thread issued so far have completed.
-__device__ __forceinline__ void commit_multicast(uint32_t mbar, uint16_t cta_mask)
-{
-    asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(mbar),
-        "h"(cta_mask)
-        : "memory");
-}
-
-__device__ __forceinline__ uint32_t cluster_ctarank()
-{
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-    return r;
 }
 
 __device__ __forceinline__ void cluster_sync()

@@ -25,3 +25,20 @@ def pytest_collection_modifyitems(config, items):
     for item in items:
         if "gpu" in item.keywords:
             item.add_marker(skip)
+
+
+@pytest.fixture
+def tuning(monkeypatch):
+    """Set GBMLA_* testing variables (attention tiling) for one test.  The
+    library reads them once per process, so each change is followed by
+    mla_reload_tuning, and the defaults are restored and re-read afterwards."""
+    from paper_2607_27269_gb300 import abi
+
+    def apply(**env):
+        for k, v in env.items():
+            monkeypatch.setenv(k, str(v))
+        abi.reload_tuning()
+
+    yield apply
+    monkeypatch.undo()
+    abi.reload_tuning()

@@ -108,13 +108,13 @@ def test_decode_step_matches_oracle(name):
 
 @pytest.mark.parametrize("kernel", ["simt", "tc"])
 @pytest.mark.parametrize("name", ["qwen05b_b16_h14_r256_t2048", "llama1b_paged_b128_h32_r512_t128_8192"])
-def test_split_count_invariance(name, kernel, monkeypatch):
+def test_split_count_invariance(name, kernel, tuning):
     """The split count changes only how the softmax sum is grouped.  The
     CUDA-core kernel keeps the weights in fp32 (agreement to fp32 noise); the
     tensor-core kernel rounds each weight to bf16 relative to the running
     maximum, which depends on where a split starts, so its bound is the bf16
     rounding of the weights (2^-9 relative each)."""
-    monkeypatch.setenv("GBMLA_ATTN_KERNEL", kernel)
+    tuning(GBMLA_ATTN_KERNEL=kernel)
     o_tol, l_tol = (1e-5, 1e-5) if kernel == "simt" else (4e-3, 1e-3)
     w = wl.small(name, seed=14)
     outs = []
@@ -217,13 +217,13 @@ def test_deterministic():
 
 
 @pytest.mark.parametrize("name", wl.ORDER)
-def test_tensor_core_kernel_matches_cuda_core_kernel(name, monkeypatch):
+def test_tensor_core_kernel_matches_cuda_core_kernel(name, tuning):
     """The two attention kernels of the library agree on the same inputs (they
     differ only in rounding: the tensor-core kernel multiplies bf16 weights)."""
     w = wl.small(name, seed=21)
     res = {}
     for kern in ("simt", "tc"):
-        monkeypatch.setenv("GBMLA_ATTN_KERNEL", kern)
+        tuning(GBMLA_ATTN_KERNEL=kern)
         step = run_step(abi.to_device(w))
         res[kern] = (step.o_lat.cpu().numpy().astype(np.float64), step.lse.cpu().numpy().astype(np.float64))
     mx, mean = rel_errors(res["tc"][0], res["simt"][0])
@@ -232,24 +232,22 @@ def test_tensor_core_kernel_matches_cuda_core_kernel(name, monkeypatch):
 
 
 @pytest.mark.parametrize("env", [
-    {},                                                   # 2 x 80 rows, cluster of two with multicast
-    {"GBMLA_TC_NO_CLUSTER": "1"},                         # 2 x 80 rows, independent CTAs
+    {},                                                   # 2 x 80 rows, independent CTAs
     {"GBMLA_TC_MAX_SLOTS": "4"},                          # the smallest ring: every slot reused within a tile
     {"GBMLA_TC_MAX_N": "32", "GBMLA_TC_MAX_SLOTS": "4"},  # 5 x 32 rows
     {"GBMLA_TC_MAX_N": "48"},
     {"GBMLA_TC_MAX_N": "64"},
-], ids=["cluster80", "nocluster80", "ring4", "n32_ring4", "n48", "n64"])
+], ids=["rows80", "ring4", "n32_ring4", "n48", "n64"])
 @pytest.mark.parametrize("splits", [1, 3, 7])
-def test_tensor_core_kernel_shapes_and_rings(env, splits, monkeypatch):
+def test_tensor_core_kernel_shapes_and_rings(env, splits, tuning):
     """Several sequences per CTA, tail tiles of one or two pages, and rings
     smaller than a tile's chunk count (the regime where a look-ahead barrier
-    wait once cleared the next sequence's rows): every query-group size,
-    cluster mode and ring size matches the oracle.  With 32 and 48 rows the
+    wait once cleared the next sequence's rows): every query-group size and
+    ring size matches the oracle.  With 32 and 48 rows the
     kernel alternates two O^T buffers between sequences and drains each after
     the next one's first tile; one split puts all five sequences in one CTA,
     so both buffers are reused and every deferred drain runs."""
-    for k, v in env.items():
-        monkeypatch.setenv(k, v)
+    tuning(**env)
     shape = wl.SHAPES["llama1b_paged_b128_h32_r512_t128_8192"]
     w = wl.make(shape, seed=15, batch=5, kv_range=(70, 650))
     step = run_step(abi.to_device(w), num_splits=splits)

@@ -96,11 +96,11 @@ def _plant(t: torch.Tensor, mask: torch.Tensor, gen: torch.Generator):
 
 @pytest.mark.parametrize("kernel", ["simt", "tc"])
 @pytest.mark.parametrize("name", ["qwen05b_b16_h14_r256_t2048", "llama1b_paged_b128_h32_r512_t128_8192"])
-def test_rows_past_kv_len_are_never_read(name, kernel, monkeypatch):
+def test_rows_past_kv_len_are_never_read(name, kernel, tuning):
     """Rows at or past a sequence's length (inside its capacity, in the tail of
     its last page, or in pages no sequence owns) hold +-1e4: every output is
     bit-identical to the run with ordinary values there."""
-    monkeypatch.setenv("GBMLA_ATTN_KERNEL", kernel)
+    tuning(GBMLA_ATTN_KERNEL=kernel)
     s = wl.SHAPES[name]
     if s.paged:
         w = wl.make(s, seed=32, batch=6, kv_range=(s.q_len + 1, 700), spare_pages=3)
@@ -121,11 +121,11 @@ def test_rows_past_kv_len_are_never_read(name, kernel, monkeypatch):
 
 
 @pytest.mark.parametrize("kernel", ["simt", "tc"])
-def test_causal_mask_inside_the_chunk(kernel, monkeypatch):
+def test_causal_mask_inside_the_chunk(kernel, tuning):
     """Query i of a chunk sees chunk tokens up to i only: replacing the last
     chunk token by +-1e4 leaves the outputs of every earlier query bit-identical
     and changes those of the last query."""
-    monkeypatch.setenv("GBMLA_ATTN_KERNEL", kernel)
+    tuning(GBMLA_ATTN_KERNEL=kernel)
     s = wl.SHAPES["llama1b_chunk5_b32_h32_r512_t4096"]
     w = wl.make(s, seed=34, batch=3, kv_range=(300, 1100))
     clean = outputs(run_step(abi.to_device(w)))
