@@ -33,7 +33,9 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-DEFAULT_WORKLOAD = "qwen05b_b16_h14_r256_t2048"
+DEFAULT_WORKLOAD = "llama1b_paged_b128_h32_r512_t128_8192"
+# the other workload the attention target names; its attention core is rated in the same run
+LONG_WORKLOAD = "llama3b_long_b8_h24_r512_t16k_32k"
 METRIC = "MLA decode-attn μs/step and latent-cache HBM GB/s (% of GB300 peak), 1 GPU"
 NOMINAL_HBM_GBS = 8000.0  # the ~8 TB/s HBM3e figure the attention target is also quoted against
 
@@ -48,6 +50,8 @@ def parse_args(argv=None):
     p.add_argument("--num-splits", type=int, default=0)
     p.add_argument("--no-graph", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-long", action="store_true",
+                   help="skip the second attention rating on the long-context workload")
     p.add_argument("--seed", type=int, default=0)
     p.add_argument("--attn-launches", type=int, default=0,
                    help="profiling aid: one full step, then this many attention launches alone; no timing")
@@ -243,26 +247,10 @@ def run_ours(args, rank, world, local):
         # ---- the attention kernel alone: a CUDA graph of back-to-back launches
         # over the replicas (no host time between them), timed with events on
         # the stream it replays on
-        n_attn = max(replicas, min(args.steps, 4 * replicas))
-        g_attn = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g_attn, stream=stream):
-            for i in range(n_attn):
-                d, st = dws[i % replicas], steps[i % replicas]
-                abi.decode_attn(d.dims, d.cache, d.kv_len, d.max_kv_len, st.q_abs, st.o_part, st.lse_part, S,
-                                stream)
-        for _ in range(2):
-            g_attn.replay()
-        torch.cuda.synchronize(dev)
-        attn_ms = []
-        reps = max(1, args.steps // n_attn)
-        for _ in range(reps):
-            a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            a0.record(stream)
-            g_attn.replay()
-            a1.record(stream)
-            attn_ms.append((a0, a1))
-        torch.cuda.synchronize(dev)
-        attn_ms = [a.elapsed_time(b) / n_attn for a, b in attn_ms]
+        attn_avg_ms = time_attention(dws, steps, S, stream, dev, args.steps)
+        long_roof = None
+        if shape.name != LONG_WORKLOAD and not args.no_long:
+            long_roof = measure_long_attention(args, rank, stream, dev, l2)
 
         proj = measure_projection(args, w, dws, stream, dev, l2, peaks=load_peaks())
         accept = measure_acceptance(args, stream, dev, l2, peaks=load_peaks())
@@ -314,17 +302,8 @@ def run_ours(args, rank, world, local):
     max_e2e = max_over_ranks(e2e_ms, world, dev)
     total_bytes = sum_over_ranks(float(cache_bytes) * args.steps, world, dev)
     ms_step = max_ms / args.steps
-    attn_avg_ms = sum(attn_ms) / len(attn_ms)
     peaks = load_peaks()
-    achieved = cache_bytes / (attn_avg_ms * 1e-3) / 1e9
-    # algorithmic flops of the attention core: per query (b, i, head) with
-    # kv_b - q + i + 1 visible keys, 2 (r + d_rope) per key for the scores and 2 r
-    # for P C
-    kv = [int(x) for x in w.kv_len.tolist()]
-    keys = sum(k - shape.q_len + i + 1 for k in kv for i in range(shape.q_len)) * shape.num_heads
-    attn_flops = float(keys) * (2 * (shape.rank + shape.d_rope) + 2 * shape.rank)
-    attn_tflops = attn_flops / (attn_avg_ms * 1e-3) / 1e12
-    t_floor = max(cache_bytes / (peaks["hbm_gbs"] * 1e9), attn_flops / (peaks["bf16_tflops"] * 1e12))
+    roof = attention_roofline(w, attn_avg_ms, peaks)
 
     def pct(q):
         return round(step_ms[min(len(step_ms) - 1, int(q * len(step_ms)))] * 1e3, 3)
@@ -357,16 +336,8 @@ def run_ours(args, rank, world, local):
                   f"{l2 / 2**20:.0f} MiB); no flush",
             "cuda_graph": graphs is not None, "parallelism": f"replicas{world}",
         },
-        "roofline": {
-            "bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
-            "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": attn_traffic(shape.name),
-            "peak_source": peaks["source"], "kernel": "mla_decode_attn",
-            "bytes_per_launch": cache_bytes,
-            "flops_per_launch": attn_flops, "achieved_tflops": round(attn_tflops, 1),
-            "tensor_frac": round(attn_tflops / peaks["bf16_tflops"], 4),
-            "ridge_frac": round(t_floor / (attn_avg_ms * 1e-3), 4),
-            "nominal_gbs": NOMINAL_HBM_GBS, "nominal_frac": round(achieved / NOMINAL_HBM_GBS, 4),
-        },
+        "roofline": roof,
+        "roofline_long": long_roof,
         "step_us_dist": {"p10": pct(0.1), "p50": pct(0.5), "p90": pct(0.9)},
         "clocks": clocks.summary(),
         "e2e": {"value": round(total_bytes / (max_e2e * 1e-3) / 1e9, 2), "unit": "GB/s",
@@ -379,6 +350,89 @@ def run_ours(args, rank, world, local):
         "e2e_loss_forward": e2e_fwd,
     }
     return line, w
+
+
+def time_attention(dws, steps, S, stream, dev, n_steps):
+    """Mean time (ms) of one attention launch (mla_decode_attn): a CUDA graph
+    of back-to-back launches over the replicas, timed with CUDA events on the
+    stream the graph replays on."""
+    import torch
+    from paper_2607_27269_gb300 import abi
+
+    replicas = len(dws)
+    n_attn = max(replicas, min(max(n_steps, 16), 4 * replicas))
+    g_attn = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_attn, stream=stream):
+        for i in range(n_attn):
+            d, st = dws[i % replicas], steps[i % replicas]
+            abi.decode_attn(d.dims, d.cache, d.kv_len, d.max_kv_len, st.q_abs, st.o_part, st.lse_part, S, stream)
+    for _ in range(2):
+        g_attn.replay()
+    torch.cuda.synchronize(dev)
+    marks = []
+    for _ in range(max(3, n_steps // n_attn)):
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        g_attn.replay()
+        a1.record(stream)
+        marks.append((a0, a1))
+    torch.cuda.synchronize(dev)
+    code = abi.check_status(stream)
+    if code != abi.MLA_OK:
+        raise RuntimeError(f"device status after the attention launches: {abi.status_name(code)}")
+    ms = [a.elapsed_time(b) / n_attn for a, b in marks]
+    return sum(ms) / len(ms)
+
+
+def attention_roofline(w, attn_ms, peaks):
+    """Roofline of the attention core on workload `w` from its mean launch
+    time: algorithmic bytes = the latent + positional cache read once for all
+    heads; algorithmic FLOPs = scores over the visible keys plus P C."""
+    shape = w.shape
+    cache_bytes = w.cache_bytes
+    achieved = cache_bytes / (attn_ms * 1e-3) / 1e9
+    # per query (b, i, head) with kv_b - q + i + 1 visible keys: 2 (r + d_rope)
+    # per key for the scores and 2 r for P C
+    kv = [int(x) for x in w.kv_len.tolist()]
+    keys = sum(k - shape.q_len + i + 1 for k in kv for i in range(shape.q_len)) * shape.num_heads
+    flops = float(keys) * (2 * (shape.rank + shape.d_rope) + 2 * shape.rank)
+    tflops = flops / (attn_ms * 1e-3) / 1e12
+    t_floor = max(cache_bytes / (peaks["hbm_gbs"] * 1e9), flops / (peaks["bf16_tflops"] * 1e12))
+    return {
+        "bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+        "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": attn_traffic(shape.name),
+        "peak_source": peaks["source"], "kernel": "mla_decode_attn", "workload": shape.name,
+        "bytes_per_launch": cache_bytes, "attn_us_per_launch": round(attn_ms * 1e3, 3),
+        "flops_per_launch": flops, "achieved_tflops": round(tflops, 1),
+        "tensor_frac": round(tflops / peaks["bf16_tflops"], 4),
+        "ridge_frac": round(t_floor / (attn_ms * 1e-3), 4),
+        "nominal_gbs": NOMINAL_HBM_GBS, "nominal_frac": round(achieved / NOMINAL_HBM_GBS, 4),
+    }
+
+
+def measure_long_attention(args, rank, stream, dev, l2):
+    """The attention core on the long-context workload, rated like the main
+    one (replicas beyond 2x L2, a CUDA graph of back-to-back launches)."""
+    import torch
+    from paper_2607_27269_gb300 import abi
+    from paper_2607_27269_gb300 import workloads as wl
+
+    w = wl.make(wl.SHAPES[LONG_WORKLOAD], seed=args.seed + rank)
+    per = (w.c_kv.numel() + w.k_rope.numel()) * 2
+    replicas = max(2, math.ceil(2 * l2 / per) + 1)
+    dws = [abi.to_device(w, dev) for _ in range(replicas)]
+    steps = [abi.DecodeStep(d.dims, d.cache, d.batch, d.q_len, d.max_kv_len, args.num_splits) for d in dws]
+    for d, st in zip(dws, steps):  # the appended entries and the absorbed queries the attention reads
+        st(d.q_nope, d.q_pe, d.kv_len, d.w_uk, d.w_uv, d.w_o, c_new=d.c_new, kr_new=d.kr_new, start_pos=d.start_pos,
+           stream=stream)
+    torch.cuda.synchronize(dev)
+    ms = time_attention(dws, steps, steps[0].num_splits, stream, dev, args.steps)
+    roof = attention_roofline(w, ms, load_peaks())
+    roof["num_splits"] = steps[0].num_splits
+    roof["replicas"] = replicas
+    del dws, steps
+    torch.cuda.empty_cache()
+    return roof
 
 
 def measure_e2e_forward(args, w, stream, dev):
