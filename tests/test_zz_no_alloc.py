@@ -64,6 +64,52 @@ def test_noalloc_matches_caller_buffer_path_twice(case):
     assert mx <= MAX_TOL and mean <= MEAN_TOL
 
 
+SCRATCH_FLOATS = (32 << 20) // 4  # the library's static array of partials
+
+
+def _fitting_splits(batch: int, rows: int, rank: int, s_auto: int) -> int:
+    """The automatic split count lowered until (batch + S - 1) partial slots
+    of rows x rank floats (plus the lse slots, rounded up to 64 floats) fit."""
+    def need(S):
+        slots = batch + S - 1
+        return slots * rows * rank + ((slots * rows + 63) // 64) * 64
+    S = s_auto
+    while S >= 1 and need(S) > SCRATCH_FLOATS:
+        S -= 1
+    return S
+
+
+def test_noalloc_lowers_the_automatic_split_count_to_fit():
+    """The full chunk workload (32 sequences of 4096 tokens, 160 query rows,
+    rank 512) needs more partial slots at the automatic split count than the
+    array holds; with num_splits = 0 the call lowers S until they fit.  Its
+    output equals, bit for bit, mla_decode_attn + mla_combine run at that lowered
+    S with caller buffers, and the automatic-S caller-buffer result within
+    tolerance -- on two calls in a row."""
+    w = wl.make("llama1b_chunk5_b32_h32_r512_t4096", seed=5)
+    dw = abi.to_device(w)
+    s = w.shape
+    ref = _reference(dw)  # automatic S, caller buffers
+    s_auto = ref.num_splits
+    s_fit = _fitting_splits(dw.batch, dw.q_len * s.num_heads, s.rank, s_auto)
+    assert 1 <= s_fit < s_auto, (s_fit, s_auto)  # the lowering branch is the one under test
+    low = abi.DecodeStep(dw.dims, dw.cache, dw.batch, dw.q_len, dw.max_kv_len, s_fit)
+    assert low.num_splits == s_fit
+    abi.decode_attn(dw.dims, dw.cache, dw.kv_len, dw.max_kv_len, ref.q_abs, low.o_part, low.lse_part, s_fit)
+    abi.combine(dw.dims, dw.batch, dw.q_len, dw.kv_len, dw.max_kv_len, low.o_part, low.lse_part, low.o_lat, low.lse,
+                s_fit)
+    assert abi.check_status() == abi.MLA_OK
+    for call in range(2):
+        o_lat = torch.full_like(ref.o_lat, float("nan"))
+        lse = torch.full_like(ref.lse, float("nan"))
+        abi.decode_attn_noalloc(dw.dims, dw.cache, dw.kv_len, dw.max_kv_len, ref.q_abs, o_lat, lse, num_splits=0)
+        assert abi.check_status() == abi.MLA_OK
+        assert torch.equal(o_lat.cpu(), low.o_lat.cpu()), f"call {call}: o_lat differs from the lowered-S path"
+        assert torch.equal(lse.cpu(), low.lse.cpu()), f"call {call}: lse differs from the lowered-S path"
+        mx, mean = rel_errors(o_lat.cpu().numpy(), ref.o_lat.cpu().numpy())
+        assert mx <= MAX_TOL and mean <= MEAN_TOL, f"call {call}: max {mx:.3e} mean {mean:.3e}"
+
+
 def test_noalloc_refuses_sizes_beyond_its_array():
     """The full paged workload needs more partial slots than the 32 MiB array
     holds even with one split per sequence: refused before any launch."""
