@@ -3,8 +3,15 @@
 // of the two softmax distributions (Eq. 9) and greedy agreement of their
 // argmaxes (Eq. 10), one vocabulary row per context.
 //
-// A row is split over a cluster of kCluster CTAs, each owning a contiguous
-// slice of the vocabulary.  When both rows' slices fit in shared memory
+// Many rows (at least kRowKernelRows): one CTA per row, rows strided over a
+// grid of two CTAs per SM.  Pass 1 streams both logit rows from HBM and marks
+// their lines evict-last, so that pass 2 reads them again from L2; a CTA moves
+// on to its next row as soon as it has written this one, so the SM's loads
+// never wait on another CTA's reductions.  Block-wide reductions run in a
+// fixed order (bit-reproducible).
+//
+// Few rows: a row is split over a cluster of kCluster CTAs, each owning a
+// contiguous slice of the vocabulary.  When both rows' slices fit in shared memory
 // (every vocabulary of the workloads, in bf16), one thread copies them in with
 // bulk copies at the start, so the whole slice is in flight at once and HBM is
 // read exactly once; both passes then read shared memory.  Otherwise the
@@ -119,6 +126,13 @@ struct Vec<float> {
         x[2] = v.z;
         x[3] = v.w;
     }
+    __device__ static void cvt(const uint4 &w, float (&x)[4])
+    {
+        x[0] = __uint_as_float(w.x);
+        x[1] = __uint_as_float(w.y);
+        x[2] = __uint_as_float(w.z);
+        x[3] = __uint_as_float(w.w);
+    }
     __device__ static float one(const float *p) { return *p; }
 };
 template <>
@@ -134,11 +148,30 @@ struct Vec<uint16_t> {
             x[2 * e + 1] = __uint_as_float(w[e] & 0xffff0000u);
         }
     }
+    __device__ static void cvt(const uint4 &v, float (&x)[8])
+    {
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            x[2 * e] = __uint_as_float(w[e] << 16);
+            x[2 * e + 1] = __uint_as_float(w[e] & 0xffff0000u);
+        }
+    }
     __device__ static float one(const uint16_t *p) { return __uint_as_float(static_cast<uint32_t>(*p) << 16); }
 };
 
+// 16 bytes from global memory with an L2 eviction policy.
+__device__ __forceinline__ uint4 ld_hint16(const void *p, uint64_t pol)
+{
+    uint4 w;
+    asm volatile("ld.global.L2::cache_hint.v4.u32 {%0, %1, %2, %3}, [%4], %5;"
+                 : "=r"(w.x), "=r"(w.y), "=r"(w.z), "=r"(w.w)
+                 : "l"(p), "l"(pol));
+    return w;
+}
+
 // Block-wide reduction of a value with `op`; every thread gets the result.
-template <typename V, typename Op>
+template <int NT = kAccThreads, typename V, typename Op>
 __device__ V block_reduce(V v, Op op, V *scratch)
 {
     for (int o = 16; o > 0; o >>= 1) {
@@ -157,7 +190,7 @@ __device__ V block_reduce(V v, Op op, V *scratch)
     if (lane == 0) scratch[warp] = v;
     __syncthreads();
     V r = scratch[0];
-    for (int w = 1; w < kAccThreads / 32; ++w) r = op(r, scratch[w]);
+    for (int w = 1; w < NT / 32; ++w) r = op(r, scratch[w]);
     return r;
 }
 
@@ -360,11 +393,115 @@ __global__ void __launch_bounds__(kAccThreads) accept_kernel(int vocab, int64_t 
         for (int k = 0; k < pieces; ++k) mbar_wait(smem_u32(&bar[k]), 0, kWaitLimitNs);
 }
 
+// ---------------------------------------------------------------- one CTA per row
+
+constexpr int kRowThreads = 512;
+constexpr int kRowUnroll = 2;      // vectors per tensor per thread in flight
+constexpr int kRowKernelRows = 128;
+
+template <typename T>
+__global__ void __launch_bounds__(kRowThreads, 2) accept_row_kernel(int rows, int vocab, int64_t stride,
+                                                                const T *__restrict__ draft,
+                                                                const T *__restrict__ target, float *alpha,
+                                                                int32_t *argmax_d, int32_t *argmax_t,
+                                                                int32_t *greedy)
+{
+    __shared__ Stat scratch_s[kRowThreads / 32];
+    __shared__ float scratch_f[kRowThreads / 32];
+    griddep_wait();
+    griddep_launch_dependents();
+    constexpr int VN = Vec<T>::n;
+    const int nvec = vocab / VN;
+    const uint64_t keep = tc::policy_evict_last(), drop = tc::policy_evict_first();
+    auto merge = [](Stat a, Stat b) { return stat_merge(a, b); };
+    for (int64_t row = blockIdx.x; row < rows; row += gridDim.x) {
+        const T *d = draft + row * stride, *t = target + row * stride;
+        // ---- pass 1: maxima, sums, argmaxes (lines kept in L2 for pass 2)
+        Stat sd{-INFINITY, 0.f, 0x7fffffff}, st{-INFINITY, 0.f, 0x7fffffff};
+        for (int v0 = threadIdx.x; v0 < nvec; v0 += kRowThreads * kRowUnroll) {
+            uint4 wd[kRowUnroll], wt[kRowUnroll];
+#pragma unroll
+            for (int u = 0; u < kRowUnroll; ++u) {
+                const int v = v0 + u * kRowThreads;
+                if (v < nvec) {
+                    wd[u] = ld_hint16(d + static_cast<int64_t>(v) * VN, keep);
+                    wt[u] = ld_hint16(t + static_cast<int64_t>(v) * VN, keep);
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < kRowUnroll; ++u) {
+                const int v = v0 + u * kRowThreads;
+                if (v < nvec) {
+                    float xd[VN], xt[VN];
+                    Vec<T>::cvt(wd[u], xd);
+                    Vec<T>::cvt(wt[u], xt);
+                    stat_vec<VN>(sd, xd, v * VN);
+                    stat_vec<VN>(st, xt, v * VN);
+                }
+            }
+        }
+        for (int i = nvec * VN + threadIdx.x; i < vocab; i += kRowThreads) {  // the row's tail
+            stat_one(sd, Vec<T>::one(d + i), i);
+            stat_one(st, Vec<T>::one(t + i), i);
+        }
+        sd = block_reduce<kRowThreads>(sd, merge, scratch_s);
+        st = block_reduce<kRowThreads>(st, merge, scratch_s);
+        const float cd = sd.m * kLog2e + log2f(sd.s), ct = st.m * kLog2e + log2f(st.s);
+        auto pmin = [&](float xd, float xt) { return ex2(fminf(fmaf(xd, kLog2e, -cd), fmaf(xt, kLog2e, -ct))); };
+        // ---- pass 2: sum of min(p_D, p_T), a last read of the lines
+        float acc = 0.f, acc2 = 0.f;
+        for (int v0 = threadIdx.x; v0 < nvec; v0 += kRowThreads * kRowUnroll) {
+            uint4 wd[kRowUnroll], wt[kRowUnroll];
+#pragma unroll
+            for (int u = 0; u < kRowUnroll; ++u) {
+                const int v = v0 + u * kRowThreads;
+                if (v < nvec) {
+                    wd[u] = ld_hint16(d + static_cast<int64_t>(v) * VN, drop);
+                    wt[u] = ld_hint16(t + static_cast<int64_t>(v) * VN, drop);
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < kRowUnroll; ++u) {
+                const int v = v0 + u * kRowThreads;
+                if (v < nvec) {
+                    float xd[VN], xt[VN];
+                    Vec<T>::cvt(wd[u], xd);
+                    Vec<T>::cvt(wt[u], xt);
+                    const float a = tree_sum<VN>([&](int e) { return pmin(xd[e], xt[e]); });
+                    if (u & 1)
+                        acc2 += a;
+                    else
+                        acc += a;
+                }
+            }
+        }
+        acc += acc2;
+        for (int i = nvec * VN + threadIdx.x; i < vocab; i += kRowThreads)
+            acc += pmin(Vec<T>::one(d + i), Vec<T>::one(t + i));
+        acc = block_reduce<kRowThreads>(acc, [](float a, float b) { return a + b; }, scratch_f);
+        if (threadIdx.x == 0) {
+            if (alpha) alpha[row] = acc;
+            if (argmax_d) argmax_d[row] = sd.idx;
+            if (argmax_t) argmax_t[row] = st.idx;
+            if (greedy) greedy[row] = sd.idx == st.idx;
+        }
+    }
+}
+
 template <typename T>
 cudaError_t launch_typed(int rows, int vocab, const void *draft, const void *target, int64_t stride, float *alpha,
                          int32_t *argmax_d, int32_t *argmax_t, int32_t *greedy, unsigned *status, cudaStream_t st)
 {
     constexpr int vn = Vec<T>::n;
+    if (rows >= kRowKernelRows) {
+        int dev = 0, sms = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        const int grid = rows < 2 * sms ? rows : 2 * sms;
+        return launch_dependent(accept_row_kernel<T>, dim3(grid), dim3(kRowThreads), 0, st, 1, rows, vocab, stride,
+                                static_cast<const T *>(draft), static_cast<const T *>(target), alpha, argmax_d,
+                                argmax_t, greedy);
+    }
     int chunk = (vocab + kCluster - 1) / kCluster;
     chunk = (chunk + vn - 1) / vn * vn;
     const uint32_t pad = (static_cast<uint32_t>(chunk) * sizeof(T) + 15u) & ~15u;
