@@ -652,12 +652,12 @@ def measure_projection(args, w, dws, stream, dev, l2, peaks):
 # DRAM bytes (read + write) per attention launch from one ncu capture of the
 # kernel source with this sha256 prefix (profiles/attn_tc_<workload>.md); a
 # kernel that has changed since reports null.
-TRAFFIC_SOURCE = "ab8ee869b4e5ce63"
+TRAFFIC_SOURCE = "8c5b33d238dc4a09"
 TRAFFIC = {
     "qwen05b_b16_h14_r256_t2048": 21208320,  # at 128 partitions
-    "llama3b_long_b8_h24_r512_t16k_32k": 232738304,
-    "llama1b_paged_b128_h32_r512_t128_8192": 689483264,
-    "llama1b_chunk5_b32_h32_r512_t4096": 163094016,
+    "llama3b_long_b8_h24_r512_t16k_32k": 233933568,
+    "llama1b_paged_b128_h32_r512_t128_8192": 706266880,
+    "llama1b_chunk5_b32_h32_r512_t4096": 164474624,
 }
 
 
