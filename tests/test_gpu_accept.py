@@ -87,6 +87,35 @@ def test_acceptance_row_stride_and_empty():
     abi.acceptance_stats(e, e)
 
 
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_acceptance_many_rows_ties_ragged_and_strided(dtype):
+    """160 rows take the one-CTA-per-row kernel (more than one row per CTA
+    on the grid of two CTAs per SM): ragged vocabularies (a tail past the last
+    whole vector), equal maxima far apart (the lowest index wins), identical
+    rows (greedy agreement, alpha = 1) and rows padded to a longer stride --
+    every row against the oracle."""
+    g = torch.Generator().manual_seed(56)
+    rows = 160
+    for vocab in (1003, 40961):
+        d = (torch.randn(rows, vocab, generator=g) * 2).to(dtype)
+        t = (torch.randn(rows, vocab, generator=g) * 2).to(dtype)
+        d[0, vocab - 1] = d[0, 0] = 30.0
+        t[1, vocab // 2] = t[1, 1] = 30.0
+        d[rows - 1, vocab - 1] = 40.0  # the maximum in the tail
+        t[7] = d[7]
+        ref = check(d, t)
+        assert ref["greedy"][7] == 1 and abs(ref["alpha_sample"][7] - 1.0) < 1e-12
+    # rows 1040 entries apart, 1001 used
+    full = (torch.randn(rows, 1040, generator=g) * 3).to(dtype).cuda()
+    full2 = (torch.randn(rows, 1040, generator=g) * 3).to(dtype).cuda()
+    dd, tt = full[:, :1001], full2[:, :1001]
+    alpha, ad, at, gr = abi.acceptance_stats(dd, tt)
+    ref = orc.acceptance(values(dd.cpu()), values(tt.cpu()))
+    assert np.array_equal(ad.cpu().numpy(), ref["argmax_draft"])
+    assert np.array_equal(at.cpu().numpy(), ref["argmax_target"])
+    assert np.abs(alpha.cpu().numpy().astype(np.float64) - ref["alpha_sample"]).max() <= ALPHA_TOL
+
+
 @pytest.mark.parametrize("name", ["qwen05b_b16_h14_r256_t2048", "llama1b_paged_b128_h32_r512_t128_8192"])
 def test_acceptance_full_rows_sampled(name):
     """Every row of the workload on the GPU (the size bench.py times); the
