@@ -337,11 +337,12 @@ mla_status mla_check_status(void *stream);
 mla_status mla_selftest_wait_timeout(int64_t limit_ns, void *stream);
 
 /* Testing aid: re-read the GBMLA_* environment variables that choose the
- * attention kernel's tiling (they are otherwise read once per process, at the
- * first call that needs them): GBMLA_ATTN_KERNEL=simt (CUDA-core attention),
+ * kernels' tiling (they are otherwise read once per process, at the first
+ * call that needs them): GBMLA_ATTN_KERNEL=simt (CUDA-core attention),
  * GBMLA_TC_MAX_N (query rows per tensor-core CTA, 16..80), GBMLA_TC_MAX_SLOTS
- * and GBMLA_TC_PV_SLOTS (ring slots).  Results are the same under every
- * setting, up to the floating-point order of the split partials.  Not
+ * and GBMLA_TC_PV_SLOTS (ring slots), GBMLA_ABSORB=persistent|gemm (the
+ * absorption kernel, where both serve the shape).  Results are the same under
+ * every setting, up to the floating-point order of the split partials.  Not
  * thread-safe against concurrent launches; the paper has no counterpart. */
 void mla_reload_tuning(void);
 

@@ -142,6 +142,8 @@ void read_tuning()
     t.tc_max_rows = env_int("GBMLA_TC_MAX_N");
     t.tc_max_slots = env_int("GBMLA_TC_MAX_SLOTS");
     t.tc_pv_slots = env_int("GBMLA_TC_PV_SLOTS");
+    const char *ab = getenv("GBMLA_ABSORB");
+    t.absorb_path = !ab ? 0 : strcmp(ab, "persistent") == 0 ? 1 : strcmp(ab, "gemm") == 0 ? 2 : 0;
     std::lock_guard<std::mutex> lock(g_mutex);
     g_tuning = t;
 }

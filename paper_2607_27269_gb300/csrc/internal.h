@@ -50,9 +50,11 @@ cudaError_t launch_attn_simt(const AttnArgs &a, cudaStream_t st);
 // mla_reload_tuning): GBMLA_ATTN_KERNEL=simt (attn_simt = 1) forces the
 // CUDA-core attention; GBMLA_TC_MAX_N caps the query rows per tensor-core CTA;
 // GBMLA_TC_MAX_SLOTS caps its ring slots and GBMLA_TC_PV_SLOTS sets the share
-// of the value-product ring.  0 means "not set".  They change tiling only.
+// of the value-product ring; GBMLA_ABSORB=persistent|gemm (absorb_path 1|2)
+// chooses the absorption kernel where both serve the shape.  0 means "not
+// set".  They change tiling only.
 struct Tuning {
-    int attn_simt, tc_max_rows, tc_max_slots, tc_pv_slots;
+    int attn_simt, tc_max_rows, tc_max_slots, tc_pv_slots, absorb_path;
 };
 const Tuning &tuning();
 void reload_tuning();

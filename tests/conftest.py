@@ -29,7 +29,7 @@ def pytest_collection_modifyitems(config, items):
 
 @pytest.fixture
 def tuning(monkeypatch):
-    """Set GBMLA_* testing variables (attention tiling) for one test.  The
+    """Set GBMLA_* testing variables (kernel tiling) for one test.  The
     library reads them once per process, so each change is followed by
     mla_reload_tuning, and the defaults are restored and re-read afterwards."""
     from paper_2607_27269_gb300 import abi

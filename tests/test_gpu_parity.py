@@ -93,6 +93,36 @@ def test_absorb_q(name):
     assert np.all(np.abs(got[..., s.rank:] - ref) <= ulp + 1e-6)
 
 
+@pytest.mark.parametrize("path", ["persistent", "gemm"])
+@pytest.mark.parametrize("shape,batch", [
+    ("llama1b_paged_b128_h32_r512_t128_8192", 128),  # 4 heads per group: 20 whole 128-row tiles per group
+    ("llama1b_paged_b128_h32_r512_t128_8192", 127),  # a 108-row tail tile
+    ("llama3b_long_b8_h24_r512_t16k_32k", 700),      # 3 heads per group (126-row tiles), d_nope 128: two K chunks
+    ("llama1b_chunk5_b32_h32_r512_t4096", 16),       # 128-column slices, a 64-row tail tile
+    ("qwen05b_b16_h14_r256_t2048", 19),              # 7 heads per group, 133 rows: a 7-row tail tile
+    ("tiny_b1_h8_r128_t256", 3),                     # one head per group
+    (wl.Shape("rank192", 5, 8, 2, 64, 32, 64, 192, 256, 2, 100, 400), 40),  # rank 192: 64-column slices
+])
+def test_absorb_q_both_kernels(shape, batch, path, tuning):
+    """The persistent absorption kernel and the grouped GEMM, each forced,
+    against the oracle: whole and ragged row tiles, every heads-per-group
+    count, one and two K chunks, 64-, 128- and 256-column slices of the
+    latent (narrower for fewer rows), and several items per CTA (the paged
+    rows)."""
+    tuning(GBMLA_ABSORB=path)
+    s = wl.SHAPES[shape] if isinstance(shape, str) else shape
+    w = wl.make(s, seed=40, batch=batch, kv_range=(s.q_len, 64))
+    dw = abi.to_device(w)
+    q_abs = torch.empty(batch, s.q_len, s.num_heads, s.rank + s.d_rope, dtype=torch.bfloat16, device="cuda")
+    abi.absorb_q(dw.dims, dw.q_nope, dw.q_pe, dw.kv_len, dw.w_uk, q_abs)
+    assert abi.check_status() == abi.MLA_OK
+    q_lat, q_rot = orc.absorb_q(dims_of(w), bits(w.q_nope), bits(w.q_pe), w.kv_len.numpy(), bits(w.w_uk))
+    got = bf16_to_f64(bits(q_abs.cpu()))
+    assert_close(got[..., :s.rank], q_lat, "q_lat")
+    ulp = 2.0 ** (np.floor(np.log2(np.maximum(np.abs(q_rot), 1e-30))) - 7)
+    assert np.all(np.abs(got[..., s.rank:] - q_rot) <= ulp + 1e-6)
+
+
 @pytest.mark.parametrize("name", wl.ORDER)
 def test_decode_step_matches_oracle(name):
     w = wl.small(name, seed=13)
