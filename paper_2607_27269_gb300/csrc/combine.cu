@@ -8,26 +8,32 @@
 namespace gbmla {
 namespace {
 
-// Block (row group, sequence b), 128 threads.  A row of o_lat is rank floats;
-// each thread owns one float4 of it (rank / 4 threads per row) in RPT rows
-// (RPT > 1 only when there are rows enough to fill the GPU anyway: it spreads
-// the per-block prologue over more work).  The partials are merged online:
-// KF partitions per step, their log-sum-exps and partial rows all loaded
-// together, the running exponent base raised when a step brings a larger one.
-// An empty partition (fewer tiles than partitions) was never written: its
-// values are loaded (the slot exists) but never used.
-constexpr int kCombineThreads = 128;
+// Block (row block, unit b), 256 threads.  A row of o_lat is rank floats;
+// each thread owns eight consecutive floats of it (two float4; rank / 8
+// threads per row).  The threads form SG slot groups of 256 / SG threads;
+// a group holds rows side by side, RPT rows per thread.  Each group merges its
+// share of the unit's partitions (k_first + sg, + SG, ...) online: KF of them
+// per step, their log-sum-exps and partial rows all loaded together, the
+// running exponent base raised when a step brings a larger one.  With SG > 1
+// (many partitions per sequence: few sequences over many SMs) the groups'
+// merge states then meet in shared memory and group 0 finishes; the per-warp
+// chain of dependent loads and exponentials is what bounds this kernel, so
+// splitting the partitions over more warps shortens it.  An empty partition
+// (fewer tiles than partitions) was never written: its values are never used.
+constexpr int kCombineThreads = 256;
 
-template <int RPT, int KF>
+template <int RPT, int KF, int SG>
 __global__ void __launch_bounds__(kCombineThreads) combine_kernel(int batch, int q_len, int H, int rank, int max_kv,
                                                                  int S, const int32_t *__restrict__ kv_len,
                                                                  const float *__restrict__ o_part,
                                                                  const float *__restrict__ lse_part, float *o_lat,
                                                                  float *lse_out, int groups)
 {
+    static_assert(SG == 1 || RPT == 1, "slot groups merge one row per thread");
     griddep_wait();
     griddep_launch_dependents();
     __shared__ int64_t red[64];
+    __shared__ float xs[SG > 1 ? kCombineThreads * 10 : 1];
     const int b = blockIdx.y;  // unit b: sequence b / groups (groups > 1: one unit per KV group)
     int64_t T, t0;
     block_tile_sums(kv_len, batch, b, q_len, max_kv, red, &T, &t0, groups);
@@ -35,68 +41,100 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(int batch, int
     if (nb == 0 || T == 0) return;  // invalid length: recorded by the attention kernel
     const int k_first = part_of_tile(t0, T, S), k_last = part_of_tile(t0 + nb - 1, T, S);
     const int rows = q_len * H;
-    const int tpr = rank / 4, rpb = kCombineThreads / tpr;
-    const int part = threadIdx.x % tpr;
-    if (threadIdx.x >= rpb * tpr) return;  // rank / 4 need not divide the block
-    const int row0 = blockIdx.x * rpb * RPT + threadIdx.x / tpr;
+    const int tpr = rank / 8, gsz = kCombineThreads / SG, rpg = gsz / tpr;
+    const int sg = threadIdx.x / gsz, t = threadIdx.x % gsz;
+    const int part = t % tpr, rr = t / tpr;
+    const bool active = rr < rpg;  // (tpr need not divide the group)
+    const int row0 = blockIdx.x * rpg * RPT + rr;
     const bool may_be_empty = T < S;  // a partition is empty only when there are fewer tiles than partitions
-    float m[RPT], wsum[RPT];
-    float4 acc[RPT];
+    float m[RPT], wsum[RPT], acc[RPT][8];
 #pragma unroll
     for (int r = 0; r < RPT; ++r) {
         m[r] = -INFINITY;
         wsum[r] = 0.f;
-        acc[r] = make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-    for (int k0 = k_first; k0 <= k_last; k0 += KF) {
-        float l[RPT][KF];
-        float4 x[RPT][KF];
 #pragma unroll
-        for (int j = 0; j < KF; ++j) {
-            const int k = k0 + j;
-            const bool live = k <= k_last && !(may_be_empty && part_begin(k, T, S) == part_begin(k + 1, T, S));
-            const int64_t slot = static_cast<int64_t>(b) + (k <= k_last ? k : k_last);
+        for (int e = 0; e < 8; ++e) acc[r][e] = 0.f;
+    }
+    if (active) {
+        for (int k0 = k_first + sg; k0 <= k_last; k0 += SG * KF) {
+            float l[RPT][KF];
+            float4 x[RPT][KF][2];
+#pragma unroll
+            for (int j = 0; j < KF; ++j) {
+                const int k = k0 + j * SG;
+                const bool in = k <= k_last;
+                const bool live = in && !(may_be_empty && part_begin(k, T, S) == part_begin(k + 1, T, S));
+                const int64_t slot = static_cast<int64_t>(b) + (in ? k : k_last);
+#pragma unroll
+                for (int r = 0; r < RPT; ++r) {
+                    const int row = row0 + r * rpg;
+                    l[r][j] = -INFINITY;
+                    x[r][j][0] = x[r][j][1] = make_float4(0.f, 0.f, 0.f, 0.f);
+                    if (in && row < rows) {
+                        const float lv = lse_part[slot * rows + row];
+                        const float4 *src = reinterpret_cast<const float4 *>(o_part + (slot * rows + row) * rank) + 2 * part;
+                        x[r][j][0] = __ldcs(src);
+                        x[r][j][1] = __ldcs(src + 1);
+                        l[r][j] = live ? lv : -INFINITY;
+                    }
+                }
+            }
 #pragma unroll
             for (int r = 0; r < RPT; ++r) {
-                const int row = row0 + r * rpb;
-                l[r][j] = -INFINITY;
-                x[r][j] = make_float4(0.f, 0.f, 0.f, 0.f);
-                if (row < rows) {
-                    const float lv = lse_part[slot * rows + row];
-                    x[r][j] = __ldcs(reinterpret_cast<const float4 *>(o_part + (slot * rows + row) * rank) + part);
-                    l[r][j] = live ? lv : -INFINITY;
+                float bm = l[r][0];
+#pragma unroll
+                for (int j = 1; j < KF; ++j) bm = fmaxf(bm, l[r][j]);
+                if (bm == -INFINITY) continue;
+                const float mn = fmaxf(m[r], bm);
+                const float sc = m[r] == -INFINITY ? 0.f : __expf(m[r] - mn);
+                m[r] = mn;
+                wsum[r] *= sc;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc[r][e] *= sc;
+#pragma unroll
+                for (int j = 0; j < KF; ++j) {
+                    if (l[r][j] == -INFINITY) continue;  // no key there, or never written
+                    const float wk = __expf(l[r][j] - mn);
+                    wsum[r] += wk;
+                    const float xv[8] = {x[r][j][0].x, x[r][j][0].y, x[r][j][0].z, x[r][j][0].w,
+                                         x[r][j][1].x, x[r][j][1].y, x[r][j][1].z, x[r][j][1].w};
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) acc[r][e] += wk * xv[e];
                 }
             }
         }
+    }
+    if constexpr (SG > 1) {
+        float *st = xs + threadIdx.x * 10;
+        st[0] = m[0];
+        st[1] = wsum[0];
 #pragma unroll
-        for (int r = 0; r < RPT; ++r) {
-            float bm = l[r][0];
+        for (int e = 0; e < 8; ++e) st[2 + e] = acc[0][e];
+        __syncthreads();
+        if (sg != 0) return;
+        float mx = m[0];
 #pragma unroll
-            for (int j = 1; j < KF; ++j) bm = fmaxf(bm, l[r][j]);
-            if (bm == -INFINITY) continue;
-            const float mn = fmaxf(m[r], bm);
-            const float sc = m[r] == -INFINITY ? 0.f : __expf(m[r] - mn);
-            m[r] = mn;
-            wsum[r] *= sc;
-            acc[r].x *= sc;
-            acc[r].y *= sc;
-            acc[r].z *= sc;
-            acc[r].w *= sc;
+        for (int g = 1; g < SG; ++g) mx = fmaxf(mx, xs[(g * gsz + t) * 10]);
+        if (mx != -INFINITY) {
+            const float s0 = __expf(m[0] - mx);  // 0 for a group that merged nothing
+            wsum[0] *= s0;
 #pragma unroll
-            for (int j = 0; j < KF; ++j) {
-                if (l[r][j] == -INFINITY) continue;  // no key there, or never written
-                const float wk = __expf(l[r][j] - mn);
-                wsum[r] += wk;
-                acc[r].x += wk * x[r][j].x;
-                acc[r].y += wk * x[r][j].y;
-                acc[r].z += wk * x[r][j].z;
-                acc[r].w += wk * x[r][j].w;
+            for (int e = 0; e < 8; ++e) acc[0][e] *= s0;
+#pragma unroll
+            for (int g = 1; g < SG; ++g) {
+                const float *o = xs + (g * gsz + t) * 10;
+                const float sc = __expf(o[0] - mx);
+                wsum[0] += sc * o[1];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc[0][e] += sc * o[2 + e];
             }
         }
+        m[0] = mx;
     }
+    if (!active) return;
 #pragma unroll
     for (int r = 0; r < RPT; ++r) {
-        const int row = row0 + r * rpb;
+        const int row = row0 + r * rpg;
         if (row >= rows) continue;
         const float inv = wsum[r] > 0.f ? 1.f / wsum[r] : 0.f;
         // output row: (b, row) for the MLA path; for groups > 1, row = i * H + head of
@@ -104,8 +142,9 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(int batch, int
         const int64_t orow = groups == 1 ? static_cast<int64_t>(b) * rows + row
                                          : (static_cast<int64_t>(b / groups) * q_len + row / H) * (groups * H) +
                                                (b % groups) * H + row % H;
-        reinterpret_cast<float4 *>(o_lat + orow * rank)[part] =
-            make_float4(acc[r].x * inv, acc[r].y * inv, acc[r].z * inv, acc[r].w * inv);
+        float4 *dst = reinterpret_cast<float4 *>(o_lat + orow * rank) + 2 * part;
+        dst[0] = make_float4(acc[r][0] * inv, acc[r][1] * inv, acc[r][2] * inv, acc[r][3] * inv);
+        dst[1] = make_float4(acc[r][4] * inv, acc[r][5] * inv, acc[r][6] * inv, acc[r][7] * inv);
         if (lse_out && part == 0) lse_out[orow] = wsum[r] > 0.f ? m[r] + logf(wsum[r]) : -INFINITY;
     }
 }
@@ -116,20 +155,27 @@ cudaError_t launch_combine(int batch, int q_len, int num_heads, int rank, int ma
                            const int32_t *kv_len, const float *o_part, const float *lse_part, float *o_lat,
                            float *lse, cudaStream_t st, int groups)
 {
-    // rank is a multiple of 64 (<= 512): rank / 4 <= 128 threads per row
-    const int tpr = rank / 4, rpb = kCombineThreads / tpr;
+    // rank is a multiple of 64 (<= 512): rank / 8 <= 64 threads per row
+    const int tpr = rank / 8;
     const int rows = q_len * num_heads;
     if (batch == 0 || rows == 0) return cudaSuccess;
-    // four rows per thread once that still leaves several blocks per SM
-    const int64_t blocks1 = static_cast<int64_t>((rows + rpb - 1) / rpb) * batch;
-    if (blocks1 >= 16 * 152) {
-        dim3 grid((rows + 4 * rpb - 1) / (4 * rpb), batch);
-        return launch_dependent(combine_kernel<4, 2>, grid, dim3(kCombineThreads), 0, st, 1, batch, q_len, num_heads,
-                                rank, max_kv, num_splits, kv_len, o_part, lse_part, o_lat, lse, groups);
+    auto go = [&](auto kernel, int rows_per_block) {
+        dim3 grid((rows + rows_per_block - 1) / rows_per_block, batch);
+        return launch_dependent(kernel, grid, dim3(kCombineThreads), 0, st, 1, batch, q_len, num_heads, rank, max_kv,
+                                num_splits, kv_len, o_part, lse_part, o_lat, lse, groups);
+    };
+    // Many partitions per unit (a few long sequences spread over the SMs):
+    // slot groups of the smallest whole number of warps that holds a row.
+    if (num_splits >= 4 * batch) {
+        const int gsz = (tpr + 31) / 32 * 32;
+        if (kCombineThreads / gsz >= 8) return go(combine_kernel<1, 4, 8>, (kCombineThreads / 8) / tpr);
+        return go(combine_kernel<1, 4, 4>, (kCombineThreads / 4) / tpr);
     }
-    dim3 grid((rows + rpb - 1) / rpb, batch);
-    return launch_dependent(combine_kernel<1, 8>, grid, dim3(kCombineThreads), 0, st, 1, batch, q_len, num_heads, rank,
-                            max_kv, num_splits, kv_len, o_part, lse_part, o_lat, lse, groups);
+    // Few partitions per unit: rows side by side, two rows per thread once
+    // that still leaves several blocks per SM
+    const int rpb = kCombineThreads / tpr;
+    if (static_cast<int64_t>((rows + rpb - 1) / rpb) * batch >= 8 * 152) return go(combine_kernel<2, 2, 1>, 2 * rpb);
+    return go(combine_kernel<1, 4, 1>, rpb);
 }
 
 }  // namespace gbmla
