@@ -12,10 +12,11 @@ CUDA graph and rotates over enough replicas of the inputs that the bytes
 touched between two reuses exceed twice the L2.  `roofline` rates the
 attention kernel (the dominant one) on its own launches, timed with CUDA
 events on its stream.  `e2e` repeats the step through the public API with the
-step's inputs copied from pinned host memory and the output read back; for a
-step of 100 us or more of device time a second stream uploads the next step's
-inputs and reads this step's output back while it computes (a serving loop's
-overlap), below that the copies stay in line.
+step's inputs copied from pinned host memory and the output read back, in the
+faster (tried briefly before the timed region) of two loops: a second stream
+uploading the next step's inputs and reading this step's output back while it
+computes (a serving loop's overlap), or the copies in line on the step's
+stream (fewer host calls, for steps too short to hide them).
 `cpu_baseline` (rank 0, N = 1) times the fp64 CPU oracle on a bounded sample.
 
 Under torchrun (N > 1) every rank runs its own replica of the workload on its
@@ -334,10 +335,20 @@ def run_ours(args, rank, world, local):
             for i in range(n):
                 e2e_step_serial(i)
 
-        # A short step is bound by the host's launch calls, and the second
-        # stream's extra calls would only add to them: below 100 us of device
-        # time per step the copies stay in line on the step's stream.
-        pipelined = elapsed_ms / args.steps >= 0.1
+        # The loop that is faster on this machine is timed: the pipelined one
+        # hides the copies behind the compute but makes more host calls per
+        # step (a second stream, its events), which a short step cannot hide
+        # (on the GB300 machine: ~80 us of host time per step against ~50 us for
+        # the loop with the copies in line on the step's stream).
+        def trial(fn, n=8):
+            fn(2)
+            torch.cuda.synchronize(dev)
+            t0 = time.perf_counter()
+            fn(n)
+            torch.cuda.synchronize(dev)
+            return time.perf_counter() - t0
+
+        pipelined = trial(e2e_run) <= trial(e2e_run_serial)
         run = e2e_run if pipelined else e2e_run_serial
         run(3)
         torch.cuda.synchronize(dev)

@@ -157,6 +157,38 @@ def test_split_count_invariance(name, kernel, tuning):
         assert np.abs(l - outs[0][1]).max() < l_tol
 
 
+@pytest.mark.parametrize("kernel", ["simt", "tc"])
+@pytest.mark.parametrize("shape,many", [
+    ("llama3b_long_b8_h24_r512_t16k_32k", 24),   # rank 512: four slot groups of 64 threads
+    ("llama3b_long_b8_h24_r512_t16k_32k", 64),   # more partitions than tiles: empty ones in every group
+    ("qwen05b_b16_h14_r256_t2048", 16),          # rank 256: eight groups of 32 threads
+    ("tiny_b1_h8_r128_t256", 9),                 # rank 128: eight groups, two rows side by side
+    (wl.Shape("rank192", 5, 8, 2, 64, 32, 64, 192, 256, 2, 100, 400), 12),  # 24 threads of each 32 hold the row
+])
+def test_combine_slot_groups(shape, many, kernel, tuning):
+    """Many partitions per sequence (at least four) take the combine whose
+    slot groups merge a row's partitions in parallel and meet in shared
+    memory; one partition takes the plain merge.  The two agree to the
+    attention kernel's split invariance, and the split run matches the
+    oracle."""
+    s = wl.SHAPES[shape] if isinstance(shape, str) else shape
+    if kernel == "tc" and s.rank % 128:
+        pytest.skip("the tensor-core kernel serves rank % 128 == 0")
+    tuning(GBMLA_ATTN_KERNEL=kernel)
+    o_tol, l_tol = (1e-5, 1e-5) if kernel == "simt" else (4e-3, 1e-3)
+    w = wl.make(s, seed=41, batch=2, kv_range=(max(s.q_len, 300), 3000))
+    ref = oracle_step(w)
+    outs = []
+    for S in (1, many):
+        step = run_step(abi.to_device(w), num_splits=S)
+        assert step.num_splits == S
+        outs.append((step.o_lat.cpu().numpy().astype(np.float64), step.lse.cpu().numpy().astype(np.float64)))
+    assert rel_errors(outs[1][0], outs[0][0])[0] < o_tol
+    assert np.abs(outs[1][1] - outs[0][1]).max() < l_tol
+    assert_close(outs[1][0], ref["o_lat"], "o_lat")
+    assert_close(outs[1][1], ref["lse"], "lse")
+
+
 def test_paged_equals_contiguous_bitwise():
     """The same logical cache, paged through a shuffled block table or laid out
     contiguously, gives bit-identical attention outputs."""
