@@ -170,9 +170,9 @@ __device__ __forceinline__ uint4 ld_hint16(const void *p, uint64_t pol)
     return w;
 }
 
-// Block-wide reduction of a value with `op`; every thread gets the result.
-template <int NT = kAccThreads, typename V, typename Op>
-__device__ V block_reduce(V v, Op op, V *scratch)
+// Reduction over the 32 lanes of a warp by shuffles; every lane gets the result.
+template <typename V, typename Op>
+__device__ __forceinline__ V warp_reduce(V v, Op op)
 {
     for (int o = 16; o > 0; o >>= 1) {
         V w;
@@ -185,13 +185,27 @@ __device__ V block_reduce(V v, Op op, V *scratch)
         }
         v = op(v, w);
     }
+    return v;
+}
+
+// Block-wide reduction of a value with `op` (identity `id`); every thread gets
+// the result.  Each warp reduces by shuffles, then warp 0 reduces the warps'
+// partials the same way and publishes the result (a fixed tree: the bits do
+// not depend on timing).  `scratch` holds NT / 32 + 1 values.
+template <int NT = kAccThreads, typename V, typename Op>
+__device__ V block_reduce(V v, Op op, V *scratch, V id)
+{
+    v = warp_reduce(v, op);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    __syncthreads();
+    __syncthreads();  // (the previous reduction's result has been read)
     if (lane == 0) scratch[warp] = v;
     __syncthreads();
-    V r = scratch[0];
-    for (int w = 1; w < NT / 32; ++w) r = op(r, scratch[w]);
-    return r;
+    if (warp == 0) {
+        V r = warp_reduce(lane < NT / 32 ? scratch[lane] : id, op);
+        if (lane == 0) scratch[NT / 32] = r;
+    }
+    __syncthreads();
+    return scratch[NT / 32];
 }
 
 __device__ __forceinline__ void bulk_load(uint32_t dst, const void *src, uint32_t bytes, uint32_t mbar)
@@ -212,8 +226,8 @@ __global__ void __launch_bounds__(kAccThreads) accept_kernel(int vocab, int64_t 
     extern __shared__ __align__(16) unsigned char acc_smem[];
     __shared__ Stat s_stat[kCluster][2];        // (draft, target) statistics of every rank, pushed here by each
     __shared__ float s_part[kCluster];          // every rank's share of the overlap (rank 0's copy is read)
-    __shared__ Stat scratch_s[kAccThreads / 32];
-    __shared__ float scratch_f[kAccThreads / 32];
+    __shared__ Stat scratch_s[kAccThreads / 32 + 1];
+    __shared__ float scratch_f[kAccThreads / 32 + 1];
     __shared__ __align__(8) uint64_t bar[kMaxPieces];
     constexpr int VN = Vec<T>::n;
     const int rank = blockIdx.x % kCluster;
@@ -307,8 +321,9 @@ __global__ void __launch_bounds__(kAccThreads) accept_kernel(int vocab, int64_t 
         stat_one(st, Vec<T>::one(gt_row + i), y0 + i);
     }
     auto merge = [](Stat a, Stat b) { return stat_merge(a, b); };
-    sd = block_reduce(sd, merge, scratch_s);
-    st = block_reduce(st, merge, scratch_s);
+    const Stat none{-INFINITY, 0.f, 0x7fffffff};
+    sd = block_reduce(sd, merge, scratch_s, none);
+    st = block_reduce(st, merge, scratch_s, none);
     // push this rank's statistics into slot [rank] of every rank, then combine
     // all slots in rank order (every CTA computes the same bits)
     asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
@@ -374,7 +389,7 @@ __global__ void __launch_bounds__(kAccThreads) accept_kernel(int vocab, int64_t 
     }
     for (int i = nvec * VN + threadIdx.x; i < n; i += kAccThreads)
         acc += pmin(Vec<T>::one(gd_row + i), Vec<T>::one(gt_row + i));
-    acc = block_reduce(acc, [](float a, float b) { return a + b; }, scratch_f);
+    acc = block_reduce(acc, [](float a, float b) { return a + b; }, scratch_f, 0.f);
     if (threadIdx.x == 0) {  // this rank's share into slot [rank] of rank 0
         uint32_t remote;
         asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(&s_part[rank])), "r"(0));
@@ -406,8 +421,8 @@ __global__ void __launch_bounds__(kRowThreads, 2) accept_row_kernel(int rows, in
                                                                 int32_t *argmax_d, int32_t *argmax_t,
                                                                 int32_t *greedy)
 {
-    __shared__ Stat scratch_s[kRowThreads / 32];
-    __shared__ float scratch_f[kRowThreads / 32];
+    __shared__ Stat scratch_s[kRowThreads / 32 + 1];
+    __shared__ float scratch_f[kRowThreads / 32 + 1];
     griddep_wait();
     griddep_launch_dependents();
     constexpr int VN = Vec<T>::n;
@@ -444,8 +459,9 @@ __global__ void __launch_bounds__(kRowThreads, 2) accept_row_kernel(int rows, in
             stat_one(sd, Vec<T>::one(d + i), i);
             stat_one(st, Vec<T>::one(t + i), i);
         }
-        sd = block_reduce<kRowThreads>(sd, merge, scratch_s);
-        st = block_reduce<kRowThreads>(st, merge, scratch_s);
+        const Stat none{-INFINITY, 0.f, 0x7fffffff};
+        sd = block_reduce<kRowThreads>(sd, merge, scratch_s, none);
+        st = block_reduce<kRowThreads>(st, merge, scratch_s, none);
         const float cd = sd.m * kLog2e + log2f(sd.s), ct = st.m * kLog2e + log2f(st.s);
         auto pmin = [&](float xd, float xt) { return ex2(fminf(fmaf(xd, kLog2e, -cd), fmaf(xt, kLog2e, -ct))); };
         // ---- pass 2: sum of min(p_D, p_T), a last read of the lines
@@ -478,7 +494,7 @@ __global__ void __launch_bounds__(kRowThreads, 2) accept_row_kernel(int rows, in
         acc += acc2;
         for (int i = nvec * VN + threadIdx.x; i < vocab; i += kRowThreads)
             acc += pmin(Vec<T>::one(d + i), Vec<T>::one(t + i));
-        acc = block_reduce<kRowThreads>(acc, [](float a, float b) { return a + b; }, scratch_f);
+        acc = block_reduce<kRowThreads>(acc, [](float a, float b) { return a + b; }, scratch_f, 0.f);
         if (threadIdx.x == 0) {
             if (alpha) alpha[row] = acc;
             if (argmax_d) argmax_d[row] = sd.idx;

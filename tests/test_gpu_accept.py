@@ -91,12 +91,12 @@ def test_acceptance_row_stride_and_empty():
 def test_acceptance_many_rows_ties_ragged_and_strided(dtype):
     """160 rows take the one-CTA-per-row kernel (more than one row per CTA
     on the grid of two CTAs per SM): ragged vocabularies (a tail past the last
-    whole vector), equal maxima far apart (the lowest index wins), identical
-    rows (greedy agreement, alpha = 1) and rows padded to a longer stride --
-    every row against the oracle."""
+    whole vector; a vocabulary shorter than one vector), equal maxima far
+    apart (the lowest index wins), identical rows (greedy agreement, alpha =
+    1) and rows padded to a longer stride -- every row against the oracle."""
     g = torch.Generator().manual_seed(56)
     rows = 160
-    for vocab in (1003, 40961):
+    for vocab in (7, 1003, 40961):
         d = (torch.randn(rows, vocab, generator=g) * 2).to(dtype)
         t = (torch.randn(rows, vocab, generator=g) * 2).to(dtype)
         d[0, vocab - 1] = d[0, 0] = 30.0
