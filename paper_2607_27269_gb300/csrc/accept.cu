@@ -113,6 +113,104 @@ __device__ __forceinline__ Stat stat_merge(Stat a, Stat b)
     return a;
 }
 
+// ---- packed forms for bf16 logits (fewer instructions per token): the
+// vector maximum on raw bf16 pairs (exact), the exponent arguments and the
+// sums of exponentials as two-wide fp32 FMAs and adds (each lane rounds as
+// the scalar instruction does).
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+__device__ __forceinline__ uint32_t bmax2(uint32_t a, uint32_t b)
+{
+    uint32_t r;
+    asm("max.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+    return r;
+}
+
+__device__ __forceinline__ uint64_t pk(float lo, float hi)
+{
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+
+__device__ __forceinline__ void upk(uint64_t v, float &lo, float &hi)
+{
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c)
+{
+    uint64_t d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b)
+{
+    uint64_t d;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+
+// both logits of a bf16 pair as a packed fp32 pair (element 2k in the low half)
+__device__ __forceinline__ uint64_t bf16x2_f32x2(uint32_t w) { return pk(bf16_lo(w), bf16_hi(w)); }
+
+// Sum of 2^(t_e) over the four packed pairs t[0..3] (a tree of packed adds).
+__device__ __forceinline__ float ex2_sum8(const uint64_t (&t)[4])
+{
+    uint64_t e[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        float a, b;
+        upk(t[q], a, b);
+        e[q] = pk(ex2(a), ex2(b));
+    }
+    const uint64_t s = add2(add2(e[0], e[1]), add2(e[2], e[3]));
+    float lo, hi;
+    upk(s, lo, hi);
+    return lo + hi;
+}
+
+// stat_vec for eight bf16 logits in their raw 16-byte vector.
+__device__ __forceinline__ void stat_bf16(Stat &a, const uint4 &v, int ybase)
+{
+    const uint32_t mw = bmax2(bmax2(v.x, v.y), bmax2(v.z, v.w));
+    const float vm = fmaxf(bf16_lo(mw), bf16_hi(mw));
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    if (vm > a.m) {
+        a.s *= ex2((a.m - vm) * kLog2e);
+        a.m = vm;
+        int e0 = 7;
+#pragma unroll
+        for (int e = 7; e >= 0; --e)
+            if (((e & 1) ? bf16_hi(w[e >> 1]) : bf16_lo(w[e >> 1])) == vm) e0 = e;
+        a.idx = ybase + e0;
+    }
+    const float nml = -(a.m * kLog2e);
+    const uint64_t L = pk(kLog2e, kLog2e), C = pk(nml, nml);
+    uint64_t t[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) t[q] = fma2(bf16x2_f32x2(w[q]), L, C);
+    a.s += ex2_sum8(t);
+}
+
+// Sum over eight bf16 token pairs of min(p_D, p_T) = 2^min(x_D log2 e - c_D, x_T log2 e - c_T).
+__device__ __forceinline__ float pmin_bf16(const uint4 &vd, const uint4 &vt, float cd, float ct)
+{
+    const uint64_t L = pk(kLog2e, kLog2e), CD = pk(-cd, -cd), CT = pk(-ct, -ct);
+    const uint32_t wd[4] = {vd.x, vd.y, vd.z, vd.w}, wt[4] = {vt.x, vt.y, vt.z, vt.w};
+    uint64_t t[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        float d0, d1, t0, t1;
+        upk(fma2(bf16x2_f32x2(wd[q]), L, CD), d0, d1);
+        upk(fma2(bf16x2_f32x2(wt[q]), L, CT), t0, t1);
+        t[q] = pk(fminf(d0, t0), fminf(d1, t1));
+    }
+    return ex2_sum8(t);
+}
+
 template <typename T>
 struct Vec;
 template <>
@@ -447,11 +545,16 @@ __global__ void __launch_bounds__(kRowThreads, 2) accept_row_kernel(int rows, in
             for (int u = 0; u < kRowUnroll; ++u) {
                 const int v = v0 + u * kRowThreads;
                 if (v < nvec) {
-                    float xd[VN], xt[VN];
-                    Vec<T>::cvt(wd[u], xd);
-                    Vec<T>::cvt(wt[u], xt);
-                    stat_vec<VN>(sd, xd, v * VN);
-                    stat_vec<VN>(st, xt, v * VN);
+                    if constexpr (sizeof(T) == 2) {
+                        stat_bf16(sd, wd[u], v * VN);
+                        stat_bf16(st, wt[u], v * VN);
+                    } else {
+                        float xd[VN], xt[VN];
+                        Vec<T>::cvt(wd[u], xd);
+                        Vec<T>::cvt(wt[u], xt);
+                        stat_vec<VN>(sd, xd, v * VN);
+                        stat_vec<VN>(st, xt, v * VN);
+                    }
                 }
             }
         }
@@ -480,10 +583,15 @@ __global__ void __launch_bounds__(kRowThreads, 2) accept_row_kernel(int rows, in
             for (int u = 0; u < kRowUnroll; ++u) {
                 const int v = v0 + u * kRowThreads;
                 if (v < nvec) {
-                    float xd[VN], xt[VN];
-                    Vec<T>::cvt(wd[u], xd);
-                    Vec<T>::cvt(wt[u], xt);
-                    const float a = tree_sum<VN>([&](int e) { return pmin(xd[e], xt[e]); });
+                    float a;
+                    if constexpr (sizeof(T) == 2) {
+                        a = pmin_bf16(wd[u], wt[u], cd, ct);
+                    } else {
+                        float xd[VN], xt[VN];
+                        Vec<T>::cvt(wd[u], xd);
+                        Vec<T>::cvt(wt[u], xt);
+                        a = tree_sum<VN>([&](int e) { return pmin(xd[e], xt[e]); });
+                    }
                     if (u & 1)
                         acc2 += a;
                     else
