@@ -22,6 +22,9 @@
  *                      (Eq. 5; the block output "after its fixed output
  *                      projection", Sec. 4.1)
  *
+ * mla_decode_step runs append (optional), absorption, attention, combine and
+ * the projections in one call.
+ *
  * Conventions shared by every entry point
  *   - All pointers except the two structs are DEVICE pointers on the current
  *     CUDA device.  The caller owns and allocates every buffer; the library
@@ -208,6 +211,22 @@ mla_status mla_combine(const mla_dims *dims, int32_t batch, int32_t q_len, int32
  * hidden == 0 skips the second product and out may then be NULL. */
 mla_status mla_out_proj(const mla_dims *dims, int32_t batch, int32_t q_len, const float *o_lat,
                         const void *w_uv, const void *w_o, void *o, void *out, void *stream);
+
+/* One decode step in one call: mla_cache_append (of q_len new entries per
+ * sequence at start_pos, when c_new is not NULL), mla_absorb_q,
+ * mla_decode_attn, mla_combine and mla_out_proj, launched in that order on
+ * `stream` with the arguments and buffers those five calls take (o_part and
+ * lse_part sized by mla_workspace_size for the same batch, q_len, max_kv_len
+ * and num_splits).  Every stage's arguments are checked before the first
+ * launch: an error returns with nothing launched.  The results are those of
+ * the five calls, bit for bit; one call instead of five saves the caller's
+ * per-call overhead on short steps.  The paper has no counterpart (it is the
+ * step of Sec. 3.2-3.3 as a whole). */
+mla_status mla_decode_step(const mla_dims *dims, const mla_cache *cache, int32_t batch, int32_t q_len,
+                           const void *c_new, const void *kr_new, const int32_t *start_pos, const void *q_nope,
+                           const void *q_pe, const int32_t *kv_len, int32_t max_kv_len, const void *w_uk,
+                           const void *w_uv, const void *w_o, int32_t num_splits, void *q_abs, float *o_part,
+                           float *lse_part, float *o_lat, float *lse, void *o, void *out, void *stream);
 
 /* Acceptance statistics of a draft against its target at the same contexts
  * (Sec. 3.3), one row per context over a vocabulary of `vocab` tokens:

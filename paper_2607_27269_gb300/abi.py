@@ -22,8 +22,8 @@ SPLIT_TILE = 128
 EXPORTS = ("mla_workspace_size", "mla_cache_append", "mla_project_append", "mla_acceptance_stats",
            "mla_gqa_append", "mla_gqa_workspace_size", "mla_gqa_decode_attn", "mla_gqa_project", "mla_gqa_out_proj",
            "mla_e2e_loss", "mla_absorb_q", "mla_decode_attn", "mla_combine",
-           "mla_out_proj", "mla_check_status", "mla_selftest_wait_timeout", "mla_decode_attn_noalloc",
-           "mla_reload_tuning", "mla_status_str", "mla_last_error")
+           "mla_out_proj", "mla_decode_step", "mla_check_status", "mla_selftest_wait_timeout",
+           "mla_decode_attn_noalloc", "mla_reload_tuning", "mla_status_str", "mla_last_error")
 
 
 class MlaError(RuntimeError):
@@ -89,6 +89,8 @@ def lib(auto_build: bool = True):
             L.mla_decode_attn.argtypes = [P(MlaDims), P(MlaCache), i32, i32, vp, i32, vp, i32, vp, vp, vp]
             L.mla_combine.argtypes = [P(MlaDims), i32, i32, i32, vp, i32, vp, vp, vp, vp, vp]
             L.mla_out_proj.argtypes = [P(MlaDims), i32, i32, vp, vp, vp, vp, vp, vp]
+            L.mla_decode_step.argtypes = [P(MlaDims), P(MlaCache), i32, i32, vp, vp, vp, vp, vp, vp, i32, vp, vp, vp,
+                                          i32, vp, vp, vp, vp, vp, vp, vp, vp]
             L.mla_check_status.argtypes = [vp]
             L.mla_selftest_wait_timeout.argtypes = [i64, vp]
             L.mla_decode_attn_noalloc.argtypes = [P(MlaDims), P(MlaCache), i32, i32, vp, i32, vp, i32, vp, vp, vp]
@@ -387,10 +389,10 @@ def selftest_wait_timeout(limit_ns: int, stream=None):
 
 
 class DecodeStep:
-    """One decode step of an MLA layer through the five entry points, with
-    every intermediate buffer allocated once (by PyTorch) up front:
-    append -> absorb -> split-KV attention -> combine -> up/out projection
-    (or, through ``from_hidden``, projection -> absorb -> ...)."""
+    """One decode step of an MLA layer (mla_decode_step: the five entry points
+    in one call), with every intermediate buffer allocated once (by PyTorch)
+    up front: append -> absorb -> split-KV attention -> combine -> up/out
+    projection (or, through ``from_hidden``, projection -> absorb -> ...)."""
 
     def __init__(self, dims: Dims, cache: Cache, batch: int, q_len: int, max_kv_len: int, num_splits: int = 0,
                  device=None):
@@ -422,18 +424,15 @@ class DecodeStep:
                            self.out.data_ptr() if self.out is not None else None)
         dims, cache, qa, op, lp, ol, ls, o, out = self._fixed
         d, L, sp = self.dims, lib(), _stream(stream)
-        B, q = self.batch, self.q_len
-        if c_new is not None:
-            _check("mla_cache_append", L.mla_cache_append(dims, cache, B, c_new.shape[1], _p(c_new), _p(kr_new),
-                                                          _p(start_pos), sp))
-        kv = _p(kv_len)
-        _check("mla_absorb_q", L.mla_absorb_q(dims, B, q, _p(q_nope), _p(q_pe), kv, _p(w_uk), qa, sp))
-        _check("mla_decode_attn", L.mla_decode_attn(dims, cache, B, q, kv, self.max_kv_len, qa, self.num_splits, op,
-                                                    lp, sp))
-        _check("mla_combine", L.mla_combine(dims, B, q, self.num_splits, kv, self.max_kv_len, op, lp, ol, ls, sp))
+        if c_new is not None and c_new.shape[1] != self.q_len:
+            raise ValueError("c_new must hold q_len new entries per sequence")
         with_o = d.hidden and w_o is not None
-        _check("mla_out_proj", L.mla_out_proj(dims, B, q, ol, _p(w_uv), _p(w_o) if with_o else None, o,
-                                              out if with_o else None, sp))
+        # the whole step in one library call (append, absorption, attention, combine, projections)
+        _check("mla_decode_step", L.mla_decode_step(dims, cache, self.batch, self.q_len, _p(c_new), _p(kr_new),
+                                                    _p(start_pos), _p(q_nope), _p(q_pe), _p(kv_len), self.max_kv_len,
+                                                    _p(w_uk), _p(w_uv), _p(w_o) if with_o else None,
+                                                    self.num_splits, qa, op, lp, ol, ls, o,
+                                                    out if with_o else None, sp))
         return self.out if with_o else self.o
 
     def from_hidden(self, h, w_dkv, w_kr, w_q, start_pos, kv_len, w_uk, w_uv, w_o=None, stream=None):

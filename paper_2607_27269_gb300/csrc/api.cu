@@ -218,6 +218,120 @@ cudaError_t launch_selftest_wait(int64_t limit_ns, unsigned *status, cudaStream_
 
 using namespace gbmla;
 
+// The five entry points of the step, each as validation followed by the
+// launch; with launch == false they only validate (mla_decode_step checks
+// every stage before it launches any).
+namespace {
+
+mla_status mla_cache_append_impl(const mla_dims *dims, const mla_cache *cache, int32_t batch, int32_t n_new,
+                                 const void *c_new, const void *kr_new, const int32_t *start_pos, void *stream, bool launch)
+{
+    mla_status s = check_dims(dims);
+    if (s != MLA_OK) return s;
+    CacheView v;
+    if ((s = check_cache(dims, cache, &v)) != MLA_OK) return s;
+    if (batch < 0 || n_new < 0 || batch > 65535 || n_new > 65535) return MLA_ERR_INVALID_ARG;
+    if (batch == 0 || n_new == 0) return MLA_OK;
+    if (!c_new || !kr_new || !start_pos || !aligned16(c_new)) return MLA_ERR_INVALID_ARG;
+    if (!launch) return MLA_OK;  // (validation only)
+    unsigned *status = nullptr;
+    if ((s = device_info(&status, nullptr)) != MLA_OK) return s;
+    return from_cuda(launch_append(*dims, v, batch, n_new, c_new, kr_new, start_pos, status,
+                                   static_cast<cudaStream_t>(stream)));
+}
+
+mla_status mla_absorb_q_impl(const mla_dims *dims, int32_t batch, int32_t q_len, const void *q_nope,
+                             const void *q_pe, const int32_t *kv_len, const void *w_uk, void *q_abs, void *stream, bool launch)
+{
+    mla_status s = check_dims(dims);
+    if (s != MLA_OK) return s;
+    if (batch < 0 || q_len < 1 || q_len > 16) return MLA_ERR_INVALID_ARG;
+    if (batch == 0) return MLA_OK;
+    if (!q_nope || !q_pe || !kv_len || !w_uk || !q_abs) return MLA_ERR_INVALID_ARG;
+    if (!aligned16(q_nope) || !aligned16(w_uk) || !aligned16(q_abs)) return MLA_ERR_INVALID_ARG;
+    if (static_cast<int64_t>(batch) * q_len > (1 << 30)) return MLA_ERR_UNSUPPORTED;
+    if (!launch) return MLA_OK;  // (validation only)
+    unsigned *status = nullptr;
+    if ((s = device_info(&status, nullptr)) != MLA_OK) return s;
+    return from_cuda(launch_absorb(*dims, batch, q_len, q_nope, q_pe, kv_len, w_uk, q_abs, status,
+                                   static_cast<cudaStream_t>(stream)));
+}
+
+mla_status mla_decode_attn_impl(const mla_dims *dims, const mla_cache *cache, int32_t batch, int32_t q_len,
+                                const int32_t *kv_len, int32_t max_kv_len, const void *q_abs, int32_t num_splits,
+                                float *o_part, float *lse_part, void *stream, bool launch)
+{
+    mla_status s = check_dims(dims);
+    if (s != MLA_OK) return s;
+    CacheView v;
+    if ((s = check_cache(dims, cache, &v)) != MLA_OK) return s;
+    if (batch < 0 || q_len < 1 || q_len > 16 || num_splits < 0 || num_splits > 65535) return MLA_ERR_INVALID_ARG;
+    if (max_kv_len < q_len || max_kv_len > cache->capacity) return MLA_ERR_INVALID_ARG;
+    if (batch == 0) return MLA_OK;
+    if (!kv_len || !q_abs || !o_part || !lse_part || !aligned16(o_part) || !aligned16(q_abs))
+        return MLA_ERR_INVALID_ARG;
+    if (!launch) return MLA_OK;  // (validation only)
+    unsigned *status = nullptr;
+    int sms = 0;
+    if ((s = device_info(&status, &sms)) != MLA_OK) return s;
+    AttnArgs a;
+    a.batch = batch;
+    a.q_len = q_len;
+    a.num_heads = dims->num_heads;
+    a.rank = dims->rank;
+    a.d_rope = dims->d_rope;
+    a.sm_scale = dims->sm_scale;
+    a.kv_len = kv_len;
+    a.max_kv = max_kv_len;
+    a.q_abs = q_abs;
+    a.num_splits = resolve_splits(dims, batch, q_len, max_kv_len, num_splits, sms);
+    a.o_part = o_part;
+    a.lse_part = lse_part;
+    a.cache = v;
+    a.status = status;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    return from_cuda(use_tc_kernel(dims) ? launch_attn_tc(a, st) : launch_attn_simt(a, st));
+}
+
+mla_status mla_combine_impl(const mla_dims *dims, int32_t batch, int32_t q_len, int32_t num_splits,
+                            const int32_t *kv_len, int32_t max_kv_len, const float *o_part, const float *lse_part,
+                            float *o_lat, float *lse, void *stream, bool launch)
+{
+    mla_status s = check_dims(dims);
+    if (s != MLA_OK) return s;
+    if (batch < 0 || q_len < 1 || q_len > 16 || num_splits < 0 || max_kv_len < q_len) return MLA_ERR_INVALID_ARG;
+    if (batch == 0) return MLA_OK;
+    if (!kv_len || !o_part || !lse_part || !o_lat || !aligned16(o_part) || !aligned16(o_lat))
+        return MLA_ERR_INVALID_ARG;
+    if (!launch) return MLA_OK;  // (validation only)
+    int sms = 0;
+    if ((s = device_info(nullptr, &sms)) != MLA_OK) return s;
+    const int S = resolve_splits(dims, batch, q_len, max_kv_len, num_splits, sms);
+    // a length above max_kv_len counts as unusable in both kernels
+    return from_cuda(launch_combine(batch, q_len, dims->num_heads, dims->rank, max_kv_len, S, kv_len, o_part,
+                                    lse_part, o_lat, lse, static_cast<cudaStream_t>(stream)));
+}
+
+mla_status mla_out_proj_impl(const mla_dims *dims, int32_t batch, int32_t q_len, const float *o_lat,
+                             const void *w_uv, const void *w_o, void *o, void *out, void *stream, bool launch)
+{
+    mla_status s = check_dims(dims);
+    if (s != MLA_OK) return s;
+    if (batch < 0 || q_len < 1 || q_len > 16) return MLA_ERR_INVALID_ARG;
+    if (batch == 0) return MLA_OK;
+    if (!o_lat || !w_uv || !o) return MLA_ERR_INVALID_ARG;
+    if (w_o && dims->hidden > 0 && !out) return MLA_ERR_INVALID_ARG;
+    if (!aligned16(o_lat) || !aligned16(w_uv) || !aligned16(o)) return MLA_ERR_INVALID_ARG;
+    if (w_o && dims->hidden > 0 && (!aligned16(w_o) || !aligned16(out))) return MLA_ERR_INVALID_ARG;
+    if (!launch) return MLA_OK;  // (validation only)
+    unsigned *status = nullptr;
+    if ((s = device_info(&status, nullptr)) != MLA_OK) return s;
+    return from_cuda(launch_out_proj(*dims, batch, q_len, o_lat, w_uv, w_o, o, out, status,
+                                     static_cast<cudaStream_t>(stream)));
+}
+
+}  // namespace
+
 extern "C" {
 
 const char *mla_status_str(mla_status s)
@@ -254,17 +368,7 @@ mla_status mla_workspace_size(const mla_dims *dims, int32_t batch, int32_t q_len
 mla_status mla_cache_append(const mla_dims *dims, const mla_cache *cache, int32_t batch, int32_t n_new,
                             const void *c_new, const void *kr_new, const int32_t *start_pos, void *stream)
 {
-    mla_status s = check_dims(dims);
-    if (s != MLA_OK) return s;
-    CacheView v;
-    if ((s = check_cache(dims, cache, &v)) != MLA_OK) return s;
-    if (batch < 0 || n_new < 0 || batch > 65535 || n_new > 65535) return MLA_ERR_INVALID_ARG;
-    if (batch == 0 || n_new == 0) return MLA_OK;
-    if (!c_new || !kr_new || !start_pos || !aligned16(c_new)) return MLA_ERR_INVALID_ARG;
-    unsigned *status = nullptr;
-    if ((s = device_info(&status, nullptr)) != MLA_OK) return s;
-    return from_cuda(launch_append(*dims, v, batch, n_new, c_new, kr_new, start_pos, status,
-                                   static_cast<cudaStream_t>(stream)));
+    return mla_cache_append_impl(dims, cache, batch, n_new, c_new, kr_new, start_pos, stream, true);
 }
 
 mla_status mla_project_append(const mla_dims *dims, const mla_cache *cache, int32_t batch, int32_t n_new,
@@ -503,87 +607,52 @@ mla_status mla_e2e_loss(int32_t rows, int32_t hidden, const void *a_mla, const v
 mla_status mla_absorb_q(const mla_dims *dims, int32_t batch, int32_t q_len, const void *q_nope, const void *q_pe,
                         const int32_t *kv_len, const void *w_uk, void *q_abs, void *stream)
 {
-    mla_status s = check_dims(dims);
-    if (s != MLA_OK) return s;
-    if (batch < 0 || q_len < 1 || q_len > 16) return MLA_ERR_INVALID_ARG;
-    if (batch == 0) return MLA_OK;
-    if (!q_nope || !q_pe || !kv_len || !w_uk || !q_abs) return MLA_ERR_INVALID_ARG;
-    if (!aligned16(q_nope) || !aligned16(w_uk) || !aligned16(q_abs)) return MLA_ERR_INVALID_ARG;
-    if (static_cast<int64_t>(batch) * q_len > (1 << 30)) return MLA_ERR_UNSUPPORTED;
-    unsigned *status = nullptr;
-    if ((s = device_info(&status, nullptr)) != MLA_OK) return s;
-    return from_cuda(launch_absorb(*dims, batch, q_len, q_nope, q_pe, kv_len, w_uk, q_abs, status,
-                                   static_cast<cudaStream_t>(stream)));
+    return mla_absorb_q_impl(dims, batch, q_len, q_nope, q_pe, kv_len, w_uk, q_abs, stream, true);
 }
 
 mla_status mla_decode_attn(const mla_dims *dims, const mla_cache *cache, int32_t batch, int32_t q_len,
                            const int32_t *kv_len, int32_t max_kv_len, const void *q_abs, int32_t num_splits,
                            float *o_part, float *lse_part, void *stream)
 {
-    mla_status s = check_dims(dims);
-    if (s != MLA_OK) return s;
-    CacheView v;
-    if ((s = check_cache(dims, cache, &v)) != MLA_OK) return s;
-    if (batch < 0 || q_len < 1 || q_len > 16 || num_splits < 0 || num_splits > 65535) return MLA_ERR_INVALID_ARG;
-    if (max_kv_len < q_len || max_kv_len > cache->capacity) return MLA_ERR_INVALID_ARG;
-    if (batch == 0) return MLA_OK;
-    if (!kv_len || !q_abs || !o_part || !lse_part || !aligned16(o_part) || !aligned16(q_abs))
-        return MLA_ERR_INVALID_ARG;
-    unsigned *status = nullptr;
-    int sms = 0;
-    if ((s = device_info(&status, &sms)) != MLA_OK) return s;
-    AttnArgs a;
-    a.batch = batch;
-    a.q_len = q_len;
-    a.num_heads = dims->num_heads;
-    a.rank = dims->rank;
-    a.d_rope = dims->d_rope;
-    a.sm_scale = dims->sm_scale;
-    a.kv_len = kv_len;
-    a.max_kv = max_kv_len;
-    a.q_abs = q_abs;
-    a.num_splits = resolve_splits(dims, batch, q_len, max_kv_len, num_splits, sms);
-    a.o_part = o_part;
-    a.lse_part = lse_part;
-    a.cache = v;
-    a.status = status;
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    return from_cuda(use_tc_kernel(dims) ? launch_attn_tc(a, st) : launch_attn_simt(a, st));
+    return mla_decode_attn_impl(dims, cache, batch, q_len, kv_len, max_kv_len, q_abs, num_splits, o_part, lse_part,
+                                stream, true);
 }
 
 mla_status mla_combine(const mla_dims *dims, int32_t batch, int32_t q_len, int32_t num_splits,
                        const int32_t *kv_len, int32_t max_kv_len, const float *o_part, const float *lse_part,
                        float *o_lat, float *lse, void *stream)
 {
-    mla_status s = check_dims(dims);
-    if (s != MLA_OK) return s;
-    if (batch < 0 || q_len < 1 || q_len > 16 || num_splits < 0 || max_kv_len < q_len) return MLA_ERR_INVALID_ARG;
-    if (batch == 0) return MLA_OK;
-    if (!kv_len || !o_part || !lse_part || !o_lat || !aligned16(o_part) || !aligned16(o_lat))
-        return MLA_ERR_INVALID_ARG;
-    int sms = 0;
-    if ((s = device_info(nullptr, &sms)) != MLA_OK) return s;
-    const int S = resolve_splits(dims, batch, q_len, max_kv_len, num_splits, sms);
-    // a length above max_kv_len counts as unusable in both kernels
-    return from_cuda(launch_combine(batch, q_len, dims->num_heads, dims->rank, max_kv_len, S, kv_len, o_part,
-                                    lse_part, o_lat, lse, static_cast<cudaStream_t>(stream)));
+    return mla_combine_impl(dims, batch, q_len, num_splits, kv_len, max_kv_len, o_part, lse_part, o_lat, lse, stream,
+                            true);
 }
 
 mla_status mla_out_proj(const mla_dims *dims, int32_t batch, int32_t q_len, const float *o_lat, const void *w_uv,
                         const void *w_o, void *o, void *out, void *stream)
 {
-    mla_status s = check_dims(dims);
-    if (s != MLA_OK) return s;
-    if (batch < 0 || q_len < 1 || q_len > 16) return MLA_ERR_INVALID_ARG;
-    if (batch == 0) return MLA_OK;
-    if (!o_lat || !w_uv || !o) return MLA_ERR_INVALID_ARG;
-    if (w_o && dims->hidden > 0 && !out) return MLA_ERR_INVALID_ARG;
-    if (!aligned16(o_lat) || !aligned16(w_uv) || !aligned16(o)) return MLA_ERR_INVALID_ARG;
-    if (w_o && dims->hidden > 0 && (!aligned16(w_o) || !aligned16(out))) return MLA_ERR_INVALID_ARG;
-    unsigned *status = nullptr;
-    if ((s = device_info(&status, nullptr)) != MLA_OK) return s;
-    return from_cuda(launch_out_proj(*dims, batch, q_len, o_lat, w_uv, w_o, o, out, status,
-                                     static_cast<cudaStream_t>(stream)));
+    return mla_out_proj_impl(dims, batch, q_len, o_lat, w_uv, w_o, o, out, stream, true);
+}
+
+mla_status mla_decode_step(const mla_dims *dims, const mla_cache *cache, int32_t batch, int32_t q_len,
+                           const void *c_new, const void *kr_new, const int32_t *start_pos, const void *q_nope,
+                           const void *q_pe, const int32_t *kv_len, int32_t max_kv_len, const void *w_uk,
+                           const void *w_uv, const void *w_o, int32_t num_splits, void *q_abs, float *o_part,
+                           float *lse_part, float *o_lat, float *lse, void *o, void *out, void *stream)
+{
+    for (int pass = 0; pass < 2; ++pass) {  // every stage validated, then every stage launched
+        const bool go = pass == 1;
+        mla_status s = MLA_OK;
+        if (c_new) s = mla_cache_append_impl(dims, cache, batch, q_len, c_new, kr_new, start_pos, stream, go);
+        if (s == MLA_OK) s = mla_absorb_q_impl(dims, batch, q_len, q_nope, q_pe, kv_len, w_uk, q_abs, stream, go);
+        if (s == MLA_OK)
+            s = mla_decode_attn_impl(dims, cache, batch, q_len, kv_len, max_kv_len, q_abs, num_splits, o_part,
+                                     lse_part, stream, go);
+        if (s == MLA_OK)
+            s = mla_combine_impl(dims, batch, q_len, num_splits, kv_len, max_kv_len, o_part, lse_part, o_lat, lse,
+                                 stream, go);
+        if (s == MLA_OK) s = mla_out_proj_impl(dims, batch, q_len, o_lat, w_uv, w_o, o, out, stream, go);
+        if (s != MLA_OK) return s;
+    }
+    return MLA_OK;
 }
 
 mla_status mla_check_status(void *stream)

@@ -189,6 +189,46 @@ def test_combine_slot_groups(shape, many, kernel, tuning):
     assert_close(outs[1][1], ref["lse"], "lse")
 
 
+@pytest.mark.parametrize("name", ["llama1b_paged_b128_h32_r512_t128_8192", "llama3b_long_b8_h24_r512_t16k_32k",
+                                  "tiny_b1_h8_r128_t256"])
+def test_decode_step_call_equals_the_five_calls(name):
+    """mla_decode_step (the step in one call, as DecodeStep makes it) and
+    the five entry points called one after another give the same bits."""
+    w = wl.small(name, seed=42)
+    dw1, dw2 = abi.to_device(w), abi.to_device(w)
+    st1 = run_step(dw1)
+    st2 = abi.DecodeStep(dw2.dims, dw2.cache, dw2.batch, dw2.q_len, dw2.max_kv_len)
+    abi.cache_append(dw2.dims, dw2.cache, dw2.c_new, dw2.kr_new, dw2.start_pos)
+    abi.absorb_q(dw2.dims, dw2.q_nope, dw2.q_pe, dw2.kv_len, dw2.w_uk, st2.q_abs)
+    abi.decode_attn(dw2.dims, dw2.cache, dw2.kv_len, dw2.max_kv_len, st2.q_abs, st2.o_part, st2.lse_part,
+                    st2.num_splits)
+    abi.combine(dw2.dims, dw2.batch, dw2.q_len, dw2.kv_len, dw2.max_kv_len, st2.o_part, st2.lse_part, st2.o_lat,
+                st2.lse, st2.num_splits)
+    abi.out_proj(dw2.dims, st2.o_lat, dw2.w_uv, dw2.w_o, st2.o, st2.out)
+    assert abi.check_status() == abi.MLA_OK
+    for a, b in ((dw1.cache.c_kv, dw2.cache.c_kv), (dw1.cache.k_rope, dw2.cache.k_rope), (st1.q_abs, st2.q_abs),
+                 (st1.o_lat, st2.o_lat), (st1.lse, st2.lse), (st1.o, st2.o)):
+        assert torch.equal(a, b)
+    if st1.out is not None:
+        assert torch.equal(st1.out, st2.out)
+
+
+def test_decode_step_checks_every_stage_before_launching():
+    """An argument only a late stage rejects (a misaligned o_lat) fails the
+    call before anything runs: the cache keeps its rows (the append, the
+    first stage, did not run)."""
+    w = wl.small("qwen05b_b16_h14_r256_t2048", seed=43)
+    dw = abi.to_device(w)
+    step = abi.DecodeStep(dw.dims, dw.cache, dw.batch, dw.q_len, dw.max_kv_len)
+    before = dw.cache.c_kv.clone()
+    step.o_lat = torch.empty(step.o_lat.numel() + 1, dtype=torch.float32, device="cuda")[1:].view(step.o_lat.shape)
+    with pytest.raises(abi.MlaError):
+        step(dw.q_nope, dw.q_pe, dw.kv_len, dw.w_uk, dw.w_uv, dw.w_o, c_new=dw.c_new, kr_new=dw.kr_new,
+             start_pos=dw.start_pos)
+    torch.cuda.synchronize()
+    assert torch.equal(dw.cache.c_kv, before)
+
+
 def test_paged_equals_contiguous_bitwise():
     """The same logical cache, paged through a shuffled block table or laid out
     contiguously, gives bit-identical attention outputs."""
