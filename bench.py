@@ -16,7 +16,9 @@ step's inputs copied from pinned host memory and the output read back, in the
 faster (tried briefly before the timed region) of two loops: a second stream
 uploading the next step's inputs and reading this step's output back while it
 computes (a serving loop's overlap), or the copies in line on the step's
-stream (fewer host calls, for steps too short to hide them).
+stream (fewer host calls, for steps too short to hide them).  The step itself
+is the public DecodeStep in its CUDA-graph mode (one graph launch per step)
+unless --no-graph.
 `cpu_baseline` (rank 0, N = 1) times the fp64 CPU oracle on a bounded sample.
 
 Under torchrun (N > 1) every rank runs its own replica of the workload on its
@@ -340,6 +342,19 @@ def run_ours(args, rank, world, local):
         # step (a second stream, its events), which a short step cannot hide
         # (on the GB300 machine: ~80 us of host time per step against ~50 us for
         # the loop with the copies in line on the step's stream).
+        # the step replays as a CUDA graph captured through the public API
+        # (DecodeStep(graph=True)) unless --no-graph: one launch per step.
+        # Each replica's graph is captured here, on its filled input buffers,
+        # so that no capture falls in a trial or the timed region.
+        for r, st in enumerate(steps):
+            st.graph = graphs is not None
+            if st.graph:
+                d, v = dws[r], views[r]
+                dev_packs[r].copy_(host_pack)
+                st(v["q_nope"], v["q_pe"], v["kv_len"], d.w_uk, d.w_uv, d.w_o, c_new=v["c_new"], kr_new=v["kr_new"],
+                   start_pos=v["start_pos"])
+        torch.cuda.synchronize(dev)
+
         def trial(fn, n=8):
             fn(2)
             torch.cuda.synchronize(dev)
@@ -405,6 +420,7 @@ def run_ours(args, rank, world, local):
         "step_us_dist": {"p10": pct(0.1), "p50": pct(0.5), "p90": pct(0.9)},
         "clocks": clocks.summary(),
         "e2e": {"value": round(total_bytes / (max_e2e * 1e-3) / 1e9, 2), "unit": "GB/s", "pipelined": pipelined,
+                "graph": graphs is not None,
                 "us_per_step": round(max_e2e / args.steps * 1e3, 3),
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": launches_per_step * args.steps,

@@ -392,10 +392,19 @@ class DecodeStep:
     """One decode step of an MLA layer (mla_decode_step: the five entry points
     in one call), with every intermediate buffer allocated once (by PyTorch)
     up front: append -> absorb -> split-KV attention -> combine -> up/out
-    projection (or, through ``from_hidden``, projection -> absorb -> ...)."""
+    projection (or, through ``from_hidden``, projection -> absorb -> ...).
+
+    ``graph=True`` replays the step as a CUDA graph: the first call with a
+    given set of input tensors (their addresses) runs the step once and
+    captures it, later calls with the same tensors replay the capture, on the
+    current stream (or ``stream``, a ``torch.cuda.Stream``).  A serving loop
+    that refills fixed input buffers pays one graph launch per step instead of
+    the launches of every kernel."""
 
     def __init__(self, dims: Dims, cache: Cache, batch: int, q_len: int, max_kv_len: int, num_splits: int = 0,
-                 device=None):
+                 device=None, graph: bool = False):
+        self.graph = graph
+        self._graphs = {}
         self.dims, self.cache = dims, cache
         self.batch, self.q_len, self.max_kv_len = batch, q_len, max_kv_len
         dev = device or cache.c_kv.device
@@ -414,6 +423,31 @@ class DecodeStep:
 
     def __call__(self, q_nope, q_pe, kv_len, w_uk, w_uv, w_o=None, c_new=None, kr_new=None, start_pos=None,
                  stream=None):
+        args = (q_nope, q_pe, kv_len, w_uk, w_uv, w_o, c_new, kr_new, start_pos)
+        if not self.graph:
+            return self._launch(*args, stream=stream)
+        if stream is not None and not isinstance(stream, torch.cuda.Stream):
+            raise ValueError("graph mode takes a torch.cuda.Stream (or None)")
+        key = tuple(0 if t is None else t.data_ptr() for t in args)
+        entry = self._graphs.get(key)
+        if entry is None:
+            self._launch(*args, stream=stream)  # the library's per-device set-up runs outside the capture
+            g = torch.cuda.CUDAGraph()
+            side = torch.cuda.Stream()
+            side.wait_stream(stream or torch.cuda.current_stream())
+            with torch.cuda.graph(g, stream=side):
+                self._launch(*args)
+            (stream or torch.cuda.current_stream()).wait_stream(side)
+            entry = self._graphs[key] = (g, args)  # the tensors stay referenced while the graph lives
+        if stream is None:
+            entry[0].replay()
+        else:
+            with torch.cuda.stream(stream):
+                entry[0].replay()
+        return self.out if (self.dims.hidden and w_o is not None) else self.o
+
+    def _launch(self, q_nope, q_pe, kv_len, w_uk, w_uv, w_o=None, c_new=None, kr_new=None, start_pos=None,
+                stream=None):
         # the layer's descriptors and the step's own buffers are fixed: marshal
         # them once, so that a step costs the five library calls and little else
         if getattr(self, "_fixed", None) is None:

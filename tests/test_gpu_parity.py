@@ -213,6 +213,34 @@ def test_decode_step_call_equals_the_five_calls(name):
         assert torch.equal(st1.out, st2.out)
 
 
+def test_decode_step_graph_mode_replays_the_same_bits():
+    """DecodeStep(graph=True) captures the step per set of input tensors and
+    replays it: each replay gives the eager step's bits, and new inputs in the
+    same buffers are picked up by the replay."""
+    w = wl.small("llama1b_paged_b128_h32_r512_t128_8192", seed=44)
+    dw1, dw2 = abi.to_device(w), abi.to_device(w)
+    eager = run_step(dw1)
+    ref_out = eager.out.clone()
+    st = abi.DecodeStep(dw2.dims, dw2.cache, dw2.batch, dw2.q_len, dw2.max_kv_len, graph=True)
+    for _ in range(3):
+        out = st(dw2.q_nope, dw2.q_pe, dw2.kv_len, dw2.w_uk, dw2.w_uv, dw2.w_o, c_new=dw2.c_new, kr_new=dw2.kr_new,
+                 start_pos=dw2.start_pos)
+        torch.cuda.synchronize()
+        assert torch.equal(out, ref_out)
+        assert torch.equal(st.o_lat, eager.o_lat)
+    assert len(st._graphs) == 1
+    # new queries written into the captured buffers: the replay computes with them
+    q2 = torch.randn(dw2.q_nope.shape, generator=torch.Generator().manual_seed(5)).to(torch.bfloat16)
+    dw1.q_nope.copy_(q2)
+    dw2.q_nope.copy_(q2)
+    eager = run_step(dw1)
+    out = st(dw2.q_nope, dw2.q_pe, dw2.kv_len, dw2.w_uk, dw2.w_uv, dw2.w_o, c_new=dw2.c_new, kr_new=dw2.kr_new,
+             start_pos=dw2.start_pos)
+    torch.cuda.synchronize()
+    assert torch.equal(out, eager.out)
+    assert abi.check_status() == abi.MLA_OK
+
+
 def test_decode_step_checks_every_stage_before_launching():
     """An argument only a late stage rejects (a misaligned o_lat) fails the
     call before anything runs: the cache keeps its rows (the append, the
