@@ -305,6 +305,24 @@ def test_edge_lengths():
         assert torch.equal(st1.o_lat[0, 0, h].cpu(), c0)
 
 
+@pytest.mark.parametrize("kernel", ["tc", "simt"])
+@pytest.mark.parametrize("name", ["llama1b_chunk5_b32_h32_r512_t4096", "llama3b_long_b8_h24_r512_t16k_32k"])
+def test_longest_query_chunk(name, kernel, tuning):
+    """q_len = 16, the most the entry points take (a catch-up chunk of
+    gamma = 15): 512 or 384 query rows per sequence (seven or five row groups
+    of the tensor-core kernel), causal inside the chunk, the absorption on its
+    persistent kernel (d_nope 64) or its grouped GEMM (d_nope 128) -- the
+    step against the oracle."""
+    tuning(GBMLA_ATTN_KERNEL=kernel)
+    s = wl.SHAPES[name]
+    w = wl.make(s, seed=45, batch=3, kv_range=(16, 700), q_len=16)
+    step = run_step(abi.to_device(w))
+    ref = oracle_step(w)
+    assert_close(step.o_lat.cpu().numpy(), ref["o_lat"], "o_lat")
+    assert_close(step.lse.cpu().numpy(), ref["lse"], "lse")
+    assert_close(bf16_to_f64(bits(step.out.cpu())), ref["out"], "out")
+
+
 def test_empty_batch_is_a_noop():
     w = wl.small("tiny_b1_h8_r128_t256")
     dw = abi.to_device(w)
