@@ -259,7 +259,8 @@ mla_status mla_absorb_q_impl(const mla_dims *dims, int32_t batch, int32_t q_len,
 
 mla_status mla_decode_attn_impl(const mla_dims *dims, const mla_cache *cache, int32_t batch, int32_t q_len,
                                 const int32_t *kv_len, int32_t max_kv_len, const void *q_abs, int32_t num_splits,
-                                float *o_part, float *lse_part, void *stream, bool launch)
+                                float *o_part, float *lse_part, void *stream, bool launch, float *o_final = nullptr,
+                                float *lse_final = nullptr)
 {
     mla_status s = check_dims(dims);
     if (s != MLA_OK) return s;
@@ -287,6 +288,8 @@ mla_status mla_decode_attn_impl(const mla_dims *dims, const mla_cache *cache, in
     a.num_splits = resolve_splits(dims, batch, q_len, max_kv_len, num_splits, sms);
     a.o_part = o_part;
     a.lse_part = lse_part;
+    a.o_final = o_final;
+    a.lse_final = lse_final;
     a.cache = v;
     a.status = status;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -295,7 +298,7 @@ mla_status mla_decode_attn_impl(const mla_dims *dims, const mla_cache *cache, in
 
 mla_status mla_combine_impl(const mla_dims *dims, int32_t batch, int32_t q_len, int32_t num_splits,
                             const int32_t *kv_len, int32_t max_kv_len, const float *o_part, const float *lse_part,
-                            float *o_lat, float *lse, void *stream, bool launch)
+                            float *o_lat, float *lse, void *stream, bool launch, bool skip_whole = false)
 {
     mla_status s = check_dims(dims);
     if (s != MLA_OK) return s;
@@ -309,7 +312,7 @@ mla_status mla_combine_impl(const mla_dims *dims, int32_t batch, int32_t q_len, 
     const int S = resolve_splits(dims, batch, q_len, max_kv_len, num_splits, sms);
     // a length above max_kv_len counts as unusable in both kernels
     return from_cuda(launch_combine(batch, q_len, dims->num_heads, dims->rank, max_kv_len, S, kv_len, o_part,
-                                    lse_part, o_lat, lse, static_cast<cudaStream_t>(stream)));
+                                    lse_part, o_lat, lse, static_cast<cudaStream_t>(stream), 1, skip_whole));
 }
 
 mla_status mla_out_proj_impl(const mla_dims *dims, int32_t batch, int32_t q_len, const float *o_lat,
@@ -638,6 +641,10 @@ mla_status mla_decode_step(const mla_dims *dims, const mla_cache *cache, int32_t
                            const void *w_uv, const void *w_o, int32_t num_splits, void *q_abs, float *o_part,
                            float *lse_part, float *o_lat, float *lse, void *o, void *out, void *stream)
 {
+    // A sequence whose tiles all fall in one partition has a one-slot merge,
+    // which only copies: the tensor-core attention writes its final rows into
+    // o_lat / lse itself and the combine skips it (the same bits either way).
+    const bool direct = dims && use_tc_kernel(dims) && lse != nullptr;
     for (int pass = 0; pass < 2; ++pass) {  // every stage validated, then every stage launched
         const bool go = pass == 1;
         mla_status s = MLA_OK;
@@ -645,10 +652,10 @@ mla_status mla_decode_step(const mla_dims *dims, const mla_cache *cache, int32_t
         if (s == MLA_OK) s = mla_absorb_q_impl(dims, batch, q_len, q_nope, q_pe, kv_len, w_uk, q_abs, stream, go);
         if (s == MLA_OK)
             s = mla_decode_attn_impl(dims, cache, batch, q_len, kv_len, max_kv_len, q_abs, num_splits, o_part,
-                                     lse_part, stream, go);
+                                     lse_part, stream, go, direct ? o_lat : nullptr, direct ? lse : nullptr);
         if (s == MLA_OK)
             s = mla_combine_impl(dims, batch, q_len, num_splits, kv_len, max_kv_len, o_part, lse_part, o_lat, lse,
-                                 stream, go);
+                                 stream, go, direct);
         if (s == MLA_OK) s = mla_out_proj_impl(dims, batch, q_len, o_lat, w_uv, w_o, o, out, stream, go);
         if (s != MLA_OK) return s;
     }

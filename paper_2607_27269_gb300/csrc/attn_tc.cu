@@ -40,6 +40,7 @@ constexpr int kHalf = 64;                 // tokens per TMA box (one page when p
 constexpr int kChunkBytes = kTile * 128;  // 128 tokens x 64 bf16 columns, SW128 K-major
 constexpr int kMaxSlots = 16;               // ring slots of both rings together
 constexpr int kSoftmaxWarps = 12;
+constexpr int kWhole = 1 << 30;             // flag bit beside a sequence index (batch < 2^30)
 constexpr int kSoftmaxBase = 128;           // first softmax thread (after two producer and two MMA warps)
 constexpr int kThreads = kSoftmaxBase + 32 * kSoftmaxWarps;
 
@@ -65,6 +66,10 @@ struct TcArgs {
     const int32_t *kv_len;
     const int32_t *block_table;
     float *o_part, *lse_part;
+    // or NULL: a sequence whose tiles all lie in one partition writes its
+    // (final) output and log-sum-exp here, at row b of [B, rows, ...], instead
+    // of its partial slot (the combine then leaves that sequence alone)
+    float *o_final, *lse_final;
     unsigned *status;
     uint64_t wait_ns;
 };
@@ -264,6 +269,21 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const float (&v)[16])
     tc::wait_st();
 }
 
+// Where sequence b's output rows and log-sum-exps go: its partial slot b + k,
+// or (whole: all its tiles in this partition, and a final buffer given) its
+// final row b.
+__device__ __forceinline__ float *out_rows(const TcArgs &a, int b, int part, bool whole)
+{
+    return whole && a.o_final ? a.o_final + static_cast<int64_t>(b) * a.rows * a.rank
+                              : a.o_part + (static_cast<int64_t>(b) + part) * a.rows * a.rank;
+}
+
+__device__ __forceinline__ float *lse_rows(const TcArgs &a, int b, int part, bool whole)
+{
+    return whole && a.lse_final ? a.lse_final + static_cast<int64_t>(b) * a.rows
+                                : a.lse_part + (static_cast<int64_t>(b) + part) * a.rows;
+}
+
 // Per-thread constants of a softmax warp.
 struct SmCtx {
     int lane, tid, quarter, half, tok, n_own, group, part, nrc, ncc, cs, n_items;
@@ -321,7 +341,7 @@ __device__ __forceinline__ void sm_block_max(const SmCtx &c, const TcArgs &a, Sh
 // in this partition was t_end_seg, in one step (one O^T buffer).
 template <int N, int KOWN>
 __device__ __forceinline__ void sm_epilogue(const SmCtx &c, const TcArgs &a, Shared<N> &ss, Bars &bars,
-                                            float (&l_part)[KOWN][16], int b, int64_t t_end_seg)
+                                            float (&l_part)[KOWN][16], int b, int64_t t_end_seg, bool whole)
 {
     sm_wait<N>(c, a, ss, &bars.pv_done[t_end_seg % kPBufs<N>], static_cast<uint32_t>((t_end_seg / kPBufs<N>) & 1));
     named_sync_softmax();
@@ -346,9 +366,8 @@ __device__ __forceinline__ void sm_epilogue(const SmCtx &c, const TcArgs &a, Sha
         ss.alpha[cc] = l > 0.f ? 1.f / l : 0.f;  // reused here as 1 / l
     }
     named_sync_softmax();
-    const int64_t slot = static_cast<int64_t>(b) + c.part;
     const int valid_cols = a.rows - c.group * N;  // columns past it are padding
-    float *out = a.o_part + (slot * a.rows + c.group * N) * a.rank + c.tok;
+    float *out = out_rows(a, b, c.part, whole) + static_cast<int64_t>(c.group) * N * a.rank + c.tok;
     for (int m = 0; m < c.nrc; ++m) {
 #pragma unroll
         for (int ob = 0; ob < KOWN; ++ob) {
@@ -368,7 +387,7 @@ __device__ __forceinline__ void sm_epilogue(const SmCtx &c, const TcArgs &a, Sha
         const int row = c.group * N + cc;
         if (row < a.rows) {
             const float l = ss.lsum[cc];
-            a.lse_part[slot * a.rows + row] = l > 0.f ? (ss.m_used[cc] + log2f(l)) * 0.69314718055994531f : -INFINITY;
+            lse_rows(a, b, c.part, whole)[row] = l > 0.f ? (ss.m_used[cc] + log2f(l)) * 0.69314718055994531f : -INFINITY;
         }
     }
     tc::fence_before_sync();
@@ -380,7 +399,7 @@ __device__ __forceinline__ void sm_epilogue(const SmCtx &c, const TcArgs &a, Sha
 // its softmax denominators (1 / l kept for the drain) and its log-sum-exp.
 template <int N, int KOWN>
 __device__ __forceinline__ void sm_close(const SmCtx &c, const TcArgs &a, Shared<N> &ss, float (&l_part)[KOWN][16],
-                                         int b)
+                                         int b, bool whole)
 {
 #pragma unroll
     for (int ob = 0; ob < KOWN; ++ob) {
@@ -399,10 +418,8 @@ __device__ __forceinline__ void sm_close(const SmCtx &c, const TcArgs &a, Shared
         const float l = ss.red[0][cc] + ss.red[1][cc] + ss.red[2][cc] + ss.red[3][cc];
         ss.inv_l[cc] = l > 0.f ? 1.f / l : 0.f;
         const int row = c.group * N + cc;
-        if (row < a.rows) {
-            const int64_t slot = static_cast<int64_t>(b) + c.part;
-            a.lse_part[slot * a.rows + row] = l > 0.f ? (ss.m_used[cc] + log2f(l)) * 0.69314718055994531f : -INFINITY;
-        }
+        if (row < a.rows)
+            lse_rows(a, b, c.part, whole)[row] = l > 0.f ? (ss.m_used[cc] + log2f(l)) * 0.69314718055994531f : -INFINITY;
     }
     named_sync_softmax();  // inv_l is complete and red is free again
 }
@@ -411,15 +428,14 @@ __device__ __forceinline__ void sm_close(const SmCtx &c, const TcArgs &a, Shared
 // last tile here was t_end_seg, from O^T buffer obuf; then the buffer is free.
 template <int N, int KOWN>
 __device__ __forceinline__ void sm_drain(const SmCtx &c, const TcArgs &a, Shared<N> &ss, BarsT<N> &bars, int b,
-                                         int64_t t_end_seg, int obuf)
+                                         int64_t t_end_seg, int obuf, bool whole)
 {
     sm_wait<N>(c, a, ss, &bars.pv_done[t_end_seg % kPBufs<N>], static_cast<uint32_t>((t_end_seg / kPBufs<N>) & 1));
     named_sync_softmax();
     if (ss.sm_fail) return;
     tc::fence_after_sync();
-    const int64_t slot = static_cast<int64_t>(b) + c.part;
     const int valid_cols = a.rows - c.group * N;  // columns past it are padding
-    float *out = a.o_part + (slot * a.rows + c.group * N) * a.rank + c.tok;
+    float *out = out_rows(a, b, c.part, whole) + static_cast<int64_t>(c.group) * N * a.rank + c.tok;
     const uint32_t o_col = c.o_col0 + static_cast<uint32_t>(obuf * 4 * N);
     for (int m = 0; m < c.nrc; ++m) {
 #pragma unroll
@@ -447,6 +463,8 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
     constexpr int NB = N / 16;
     constexpr int KOWN = (NB + 2) / 3;
     float l_part[KOWN][16];
+    // the sequence open here, with kWhole set when all its tiles lie in this
+    // partition (its rows then go to the final buffers, when given)
     int b_cur = -1;
     int u = -1;  // sequences begun here (the PV warp counts the same ones)
     int64_t t_prev = -1;  // the previous tile (one O^T buffer: the drain runs at the next sequence's first tile)
@@ -467,11 +485,11 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
         if (first) {
             if constexpr (kOBufs<N> == 1) {
                 if (b_cur >= 0) {
-                    sm_epilogue<N, KOWN>(c, a, ss, bars, l_part, b_cur, t_prev);
+                    sm_epilogue<N, KOWN>(c, a, ss, bars, l_part, b_cur & ~kWhole, t_prev, (b_cur & kWhole) != 0);
                     if (ss.sm_fail) break;
                 }
             }
-            b_cur = b;
+            b_cur = b | (w.seq_start >= w.t_begin && w.seq_start + w.nb <= w.t_end ? kWhole : 0);
             ++u;
 #pragma unroll
             for (int ob = 0; ob < KOWN; ++ob)
@@ -615,7 +633,7 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
                 }
                 if (k == 1 && last) {
                     named_sync_softmax();
-                    sm_close<N, KOWN>(c, a, ss, l_part, b_cur);
+                    sm_close<N, KOWN>(c, a, ss, l_part, b_cur & ~kWhole, (b_cur & kWhole) != 0);
                     if (!w.last_of_partition()) {
                         d_b = b_cur;
                         d_t = static_cast<int>(t);
@@ -628,7 +646,7 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
                 }
                 if (db >= 0) {
                     named_sync_softmax();
-                    sm_drain<N, KOWN>(c, a, ss, bars, db, dt, dbuf);
+                    sm_drain<N, KOWN>(c, a, ss, bars, db & ~kWhole, dt, dbuf, (db & kWhole) != 0);
                     if (ss.sm_fail) break;
                 }
             }
@@ -637,7 +655,8 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
     }
     named_sync_softmax();
     if constexpr (kOBufs<N> == 1) {
-        if (b_cur >= 0 && !ss.sm_fail) sm_epilogue<N, KOWN>(c, a, ss, bars, l_part, b_cur, t_prev);
+        if (b_cur >= 0 && !ss.sm_fail)
+            sm_epilogue<N, KOWN>(c, a, ss, bars, l_part, b_cur & ~kWhole, t_prev, (b_cur & kWhole) != 0);
     }
 }
 
@@ -1086,6 +1105,8 @@ cudaError_t launch_cfg(const AttnArgs &a, int groups, cudaStream_t st)
     t.block_table = c.block_table;
     t.o_part = a.o_part;
     t.lse_part = a.lse_part;
+    t.o_final = a.o_final;
+    t.lse_final = a.lse_final;
     t.status = a.status;
     t.wait_ns = kWaitLimitNs;
     return launch_dependent(attn_tc_kernel<N>, dim3(groups, a.num_splits, 1), dim3(kThreads), smem, st, 1, t, mc,

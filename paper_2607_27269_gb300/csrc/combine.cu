@@ -27,7 +27,7 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(int batch, int
                                                                  int S, const int32_t *__restrict__ kv_len,
                                                                  const float *__restrict__ o_part,
                                                                  const float *__restrict__ lse_part, float *o_lat,
-                                                                 float *lse_out, int groups)
+                                                                 float *lse_out, int groups, int skip_whole)
 {
     static_assert(SG == 1 || RPT == 1, "slot groups merge one row per thread");
     griddep_wait();
@@ -40,6 +40,7 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(int batch, int
     const int64_t nb = seq_tiles(kv_len[b / groups], q_len, max_kv);
     if (nb == 0 || T == 0) return;  // invalid length: recorded by the attention kernel
     const int k_first = part_of_tile(t0, T, S), k_last = part_of_tile(t0 + nb - 1, T, S);
+    if (skip_whole && k_first == k_last) return;  // its one partition wrote the final rows itself
     const int rows = q_len * H;
     const int tpr = rank / 8, gsz = kCombineThreads / SG, rpg = gsz / tpr;
     const int sg = threadIdx.x / gsz, t = threadIdx.x % gsz;
@@ -153,7 +154,7 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(int batch, int
 
 cudaError_t launch_combine(int batch, int q_len, int num_heads, int rank, int max_kv, int num_splits,
                            const int32_t *kv_len, const float *o_part, const float *lse_part, float *o_lat,
-                           float *lse, cudaStream_t st, int groups)
+                           float *lse, cudaStream_t st, int groups, bool skip_whole)
 {
     // rank is a multiple of 64 (<= 512): rank / 8 <= 64 threads per row
     const int tpr = rank / 8;
@@ -162,7 +163,7 @@ cudaError_t launch_combine(int batch, int q_len, int num_heads, int rank, int ma
     auto go = [&](auto kernel, int rows_per_block) {
         dim3 grid((rows + rows_per_block - 1) / rows_per_block, batch);
         return launch_dependent(kernel, grid, dim3(kCombineThreads), 0, st, 1, batch, q_len, num_heads, rank, max_kv,
-                                num_splits, kv_len, o_part, lse_part, o_lat, lse, groups);
+                                num_splits, kv_len, o_part, lse_part, o_lat, lse, groups, skip_whole ? 1 : 0);
     };
     // Many partitions per unit (a few long sequences spread over the SMs):
     // slot groups of the smallest whole number of warps that holds a row.

@@ -26,6 +26,11 @@ struct AttnArgs {
     const void *q_abs;      // bf16 [B, q, H, rank + d_rope]
     int32_t num_splits;     // S (resolved)
     float *o_part, *lse_part;
+    // tensor-core kernel only, or NULL: a sequence whose tiles all lie in one
+    // partition writes its final output / log-sum-exp rows here ([B, q, H, rank]
+    // and [B, q, H], as mla_combine writes them) instead of its partial slot;
+    // the combine then skips it (launch_combine's skip_whole)
+    float *o_final = nullptr, *lse_final = nullptr;
     CacheView cache;
     unsigned *status;
 };
@@ -73,7 +78,7 @@ cudaError_t launch_attn_tc(const AttnArgs &a, cudaStream_t st);
 // of row (sequence, i) of o_lat / lse, i.e. [B, q_len, G * num_heads, rank].
 cudaError_t launch_combine(int batch, int q_len, int num_heads, int rank, int max_kv, int num_splits,
                            const int32_t *kv_len, const float *o_part, const float *lse_part, float *o_lat,
-                           float *lse, cudaStream_t st, int groups = 1);
+                           float *lse, cudaStream_t st, int groups = 1, bool skip_whole = false);
 
 cudaError_t launch_out_proj(const mla_dims &d, int batch, int q_len, const float *o_lat, const void *w_uv,
                             const void *w_o, void *o, void *out, unsigned *status, cudaStream_t st);
