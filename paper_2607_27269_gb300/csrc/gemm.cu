@@ -778,9 +778,24 @@ cudaError_t launch_project(const mla_dims &d, const CacheView &c, int batch, int
 {
     if (batch <= 0 || n_new <= 0) return cudaSuccess;
     // 128-column tiles once there are enough rows to be tensor-bound and the
-    // latent splits into whole 128-column tiles; 64 otherwise
-    if (batch * n_new > 32 && d.rank % 128 == 0)
+    // latent splits into whole 128-column tiles; 64 otherwise.  256-column
+    // tiles when they take fewer waves of CTAs by more than their extra bytes
+    // per K chunk (A 16 KB + B 32 KB against 16 + 16): the row tiles times the
+    // column tiles just past one wave at 128 (640 rows: 185 CTAs -> 95).
+    const int rows = batch * n_new;
+    if (rows > 32 && d.rank % 128 == 0) {
+        if (d.rank % 256 == 0) {
+            int dev = 0, sms = 0;
+            cudaGetDevice(&dev);
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+            const int nq = w_q ? d.num_heads * (d.d_nope + d.d_rope) : 0;
+            const int64_t mt = (rows + 127) / 128;
+            auto waves = [&](int bn) { return (mt * (d.rank / bn + 1 + (nq + bn - 1) / bn) + sms - 1) / sms; };
+            if (sms > 0 && waves(256) * 48 < waves(128) * 32)
+                return launch_proj<256>(d, c, batch, n_new, h, w_dkv, w_kr, w_q, start_pos, q_nope, q_pe, status, st);
+        }
         return launch_proj<128>(d, c, batch, n_new, h, w_dkv, w_kr, w_q, start_pos, q_nope, q_pe, status, st);
+    }
     return launch_proj<64>(d, c, batch, n_new, h, w_dkv, w_kr, w_q, start_pos, q_nope, q_pe, status, st);
 }
 

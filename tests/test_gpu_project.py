@@ -141,6 +141,8 @@ def test_projection_matches_oracle(name):
     ("qwen05b_b16_h14_r256_t2048", 129),          # 129 rows: 128-column tiles, a one-row tail tile
     ("llama1b_paged_b128_h32_r512_t128_8192", 40),  # 200 rows of 5-token chunks, paged
     ("llama3b_long_b8_h24_r512_t16k_32k", 33),    # 33 rows, 192-wide query heads
+    ("llama1b_paged_b128_h32_r512_t128_8192", 128),  # 640 rows: 256-column tiles (one wave of 95 CTAs)
+    ("llama1b_paged_b128_h32_r512_t128_8192", 127),  # 635 rows: 256-column tiles, a 123-row tail tile
 ])
 def test_projection_row_tiles(name, batch):
     s = wl.SHAPES[name]
