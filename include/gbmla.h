@@ -359,8 +359,10 @@ mla_status mla_selftest_wait_timeout(int64_t limit_ns, void *stream);
  * kernels' tiling (they are otherwise read once per process, at the first
  * call that needs them): GBMLA_ATTN_KERNEL=simt (CUDA-core attention),
  * GBMLA_TC_MAX_N (query rows per tensor-core CTA, 16..80), GBMLA_TC_MAX_SLOTS
- * and GBMLA_TC_PV_SLOTS (ring slots), GBMLA_ABSORB=persistent|gemm (the
- * absorption kernel, where both serve the shape).  Results are the same under
+ * and GBMLA_TC_PV_SLOTS (ring slots), GBMLA_TC_QUERY=resident|streamed (an
+ * 80-row tensor-core CTA keeps its queries in shared memory or loads them with
+ * each cache chunk), GBMLA_ABSORB=persistent|gemm (the absorption kernel, where
+ * both serve the shape).  Results are the same under
  * every setting, up to the floating-point order of the split partials.  Not
  * thread-safe against concurrent launches; the paper has no counterpart. */
 void mla_reload_tuning(void);

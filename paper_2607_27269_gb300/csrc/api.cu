@@ -144,6 +144,8 @@ void read_tuning()
     t.tc_pv_slots = env_int("GBMLA_TC_PV_SLOTS");
     const char *ab = getenv("GBMLA_ABSORB");
     t.absorb_path = !ab ? 0 : strcmp(ab, "persistent") == 0 ? 1 : strcmp(ab, "gemm") == 0 ? 2 : 0;
+    const char *tq = getenv("GBMLA_TC_QUERY");
+    t.tc_query = !tq ? 0 : strcmp(tq, "resident") == 0 ? 1 : strcmp(tq, "streamed") == 0 ? 2 : 0;
     std::lock_guard<std::mutex> lock(g_mutex);
     g_tuning = t;
 }

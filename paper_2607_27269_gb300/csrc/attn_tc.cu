@@ -660,8 +660,12 @@ __device__ __forceinline__ void softmax_role(const SmCtx &c, const TcArgs &a, Sh
     }
 }
 
-// N: query rows per CTA (multiple of 16, <= 80).
-template <int N>
+// N: query rows per CTA (multiple of 16, <= 80).  SQ (streamed queries): no
+// resident query buffer; each QK-ring slot holds a cache chunk and, behind it,
+// the query chunk that multiplies it, loaded with it from L2.  The ring then
+// gets the shared memory the resident queries held, so that more cache bytes
+// are in flight per SM, at the price of re-reading the queries once per tile.
+template <int N, bool SQ>
 __global__ void __maxnreg__(128)
     attn_tc_kernel(const __grid_constant__ TcArgs a, const __grid_constant__ CUtensorMap map_c,
                    const __grid_constant__ CUtensorMap map_r, const __grid_constant__ CUtensorMap map_q)
@@ -678,9 +682,11 @@ __global__ void __maxnreg__(128)
     const int nqc = ncc + 1;        // chunks of a tile in the QK pass: positional keys, then latent
     const int CA = a.qk_slots;      // QK ring slots
     const int CB = a.pv_slots;      // PV ring slots (even)
-    unsigned char *q_buf = smem;                                          // nqc x [N x 128 B]
-    unsigned char *ring_a = q_buf + ((nqc * N * 128 + 1023) & ~1023);     // CA x [128 x 128 B]
-    unsigned char *ring_b = ring_a + CA * kChunkBytes;                    // CB x [128 x 128 B]
+    static_assert(!SQ || (N * 128) % 1024 == 0, "a streamed query chunk keeps the slots 1024-byte aligned");
+    constexpr int kSlotA = SQ ? kChunkBytes + N * 128 : kChunkBytes;       // QK-ring slot
+    unsigned char *q_buf = smem;                                          // nqc x [N x 128 B] (resident queries)
+    unsigned char *ring_a = SQ ? smem : q_buf + ((nqc * N * 128 + 1023) & ~1023);  // CA x [kSlotA]
+    unsigned char *ring_b = ring_a + CA * kSlotA;                         // CB x [128 x 128 B]
     unsigned char *p_buf = ring_b + CB * kChunkBytes;                     // NP x NB x [128 tok x 32 B]
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -769,7 +775,7 @@ __global__ void __maxnreg__(128)
             }
             enum { kQK, kPV, kQuery, kIdle };
             const int kind = warp == 3 ? (lane < CB ? kPV : kIdle)
-                                       : (lane < CA ? kQK : (lane >= 16 && lane < 16 + nqc) ? kQuery : kIdle);
+                                       : (lane < CA ? kQK : (!SQ && lane >= 16 && lane < 16 + nqc) ? kQuery : kIdle);
             const int slot = lane;
             const int per_tile = kind == kQK ? nqc : ncc;
             const int ring_len = kind == kQK ? CA : CB;
@@ -781,14 +787,19 @@ __global__ void __maxnreg__(128)
             bool has = (kind == kQK || kind == kPV) ? c < total : kind == kQuery;
             bool ok = true;
             uint64_t wait_t0 = 0;
-            bool q_pending = kind == kQuery;  // griddepcontrol.wait still to do before the first query load
+            // griddepcontrol.wait still to do before the first query load
+            bool q_pending = SQ ? kind == kQK : kind == kQuery;
+            // streamed queries: the query box of the chunk issued in the first
+            // pass, which waits for that pass's griddepcontrol.wait
+            bool q_owed = false;
+            int q_owed_x = 0, q_owed_y = 0;
             bool first_pass = true;           // the ring lanes issue their first cache loads in it
             const uint64_t pol_keep = tc::policy_evict_last(), pol_drop = tc::policy_evict_first();
             uint32_t wbar = 0, fbar = 0, dst = 0;
             if (kind == kQK) {
                 wbar = smem_u32(&bars.qk_empty[slot]);
                 fbar = smem_u32(&bars.qk_full[slot]);
-                dst = smem_u32(ring_a + slot * kChunkBytes);
+                dst = smem_u32(ring_a + slot * kSlotA);
             } else if (kind == kPV) {
                 wbar = smem_u32(&bars.pv_empty[slot]);
                 fbar = smem_u32(&bars.pv_full[slot]);
@@ -800,14 +811,19 @@ __global__ void __maxnreg__(128)
             }
             while (true) {
                 if (kind == kQuery) has = has && !w.done();
-                if (!__any_sync(0xffffffffu, has && ok)) break;
+                if (!__any_sync(0xffffffffu, (has || q_owed) && ok)) break;
                 if (any_abort()) break;
                 bool progressed = false;
                 if (q_pending && !first_pass) {
                     griddep_wait();
                     q_pending = false;
+                    if (SQ && q_owed) {
+                        tc::tma_load_2d_hint(dst + kChunkBytes, &map_q, q_owed_x, q_owed_y, fbar, pol_keep);
+                        q_owed = false;
+                        progressed = true;
+                    }
                 }
-                if (has && ok && !q_pending) {
+                if (has && ok && !(kind == kQuery && q_pending)) {
                     const bool ready = k == 0 || mbar_test(wbar, static_cast<uint32_t>((k - 1) & 1));
                     if (!ready) {
                         const uint64_t now = global_ns();
@@ -834,13 +850,27 @@ __global__ void __maxnreg__(128)
                             const bool keys = kind == kQK && i == 0;
                             const CUtensorMap *map = keys ? &map_r : &map_c;
                             const int col = keys ? 0 : 64 * (kind == kQK ? i - 1 : i);
-                            tc::mbar_arrive_expect_tx(fbar, L.bytes);
+                            const bool sq = SQ && kind == kQK;
+                            tc::mbar_arrive_expect_tx(fbar, L.bytes + (sq ? N * 128 : 0));
                             // the QK pass keeps latent lines in L2 for the PV pass, which reads
                             // them a last time; the positional keys are read once
                             const uint64_t pol = (kind == kQK && !keys) ? pol_keep : pol_drop;
                             for (int h = 0; h < L.nh; ++h)
                                 tc::tma_load_3d_hint(dst + h * kHalf * 128, map, col, L.tok0[h], L.blk[h], fbar,
                                                      pol);
+                            if (sq) {
+                                // the query columns this chunk multiplies: the positional
+                                // part behind the latent part in each query row
+                                const int qx = 64 * (keys ? ncc : i - 1);
+                                const int qy = w.b * a.rows + group * N;
+                                if (q_pending) {
+                                    q_owed = true;
+                                    q_owed_x = qx;
+                                    q_owed_y = qy;
+                                } else {
+                                    tc::tma_load_2d_hint(dst + kChunkBytes, &map_q, qx, qy, fbar, pol_keep);
+                                }
+                            }
                             c += ring_len;
                             has = c < total;
                         }
@@ -890,7 +920,7 @@ __global__ void __maxnreg__(128)
                 int seg = -1;
                 for (int t = 0; t < n_items && ok; ++t, w.next()) {
                     if (any_abort()) break;
-                    if (w.first()) {
+                    if (!SQ && w.first()) {
                         ++seg;
                         if (!wait(&bars.q_full, seg & 1)) break;
                     }
@@ -900,8 +930,8 @@ __global__ void __maxnreg__(128)
                     for (int i = 0; i < nqc && ok; ++i) {
                         if (!wait(&bars.qk_full[rp.slot], rp.round & 1)) break;
                         tc::fence_after_sync();
-                        const uint32_t cb = ring_base + rp.slot * kChunkBytes;
-                        const uint32_t qb = q_base + (i == 0 ? ncc : i - 1) * N * 128;
+                        const uint32_t cb = ring_base + rp.slot * kSlotA;
+                        const uint32_t qb = SQ ? cb + kChunkBytes : q_base + (i == 0 ? ncc : i - 1) * N * 128;
 #pragma unroll
                         for (int kk = 0; kk < 4; ++kk)
                             tc::mma_bf16_elect(d_s, with_addr(dq, cb + kk * 32), with_addr(dq, qb + kk * 32), id_qk,
@@ -911,7 +941,7 @@ __global__ void __maxnreg__(128)
                     }
                     if (!ok) break;
                     tc::commit_elect(smem_u32(&bars.s_full[sb]));
-                    if (w.last()) tc::commit_elect(smem_u32(&bars.q_free));
+                    if (!SQ && w.last()) tc::commit_elect(smem_u32(&bars.q_free));
                 }
             } else {
                 const uint32_t id_pv = tc::idesc_bf16_f32(128, N, true, true);
@@ -1042,7 +1072,7 @@ cudaError_t encode_cache_map(CUtensorMap *m, const void *base, int cols, int64_t
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-template <int N>
+template <int N, bool SQ>
 cudaError_t launch_cfg(const AttnArgs &a, int groups, cudaStream_t st)
 {
     cudaError_t e = get_encoder();
@@ -1067,23 +1097,32 @@ cudaError_t launch_cfg(const AttnArgs &a, int groups, cudaStream_t st)
         if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
     }
     const int ncc = a.rank / 64;
-    const int q_bytes = (((ncc + 1) * N * 128) + 1023) & ~1023;
+    const int q_bytes = SQ ? 0 : (((ncc + 1) * N * 128) + 1023) & ~1023;
+    const int slot_a = SQ ? kChunkBytes + N * 128 : kChunkBytes;  // QK-ring slot (with its query chunk)
     const int p_bytes = kPBufs<N> * (N / 16) * kTile * 32;
     const int fixed = 1024 /*alignment slack*/ + q_bytes;
     int dev = 0, optin = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
     const int static_bytes = static_cast<int>(sizeof(BarsT<N>) + sizeof(Shared<N>) + 32 * 8) + 128;
-    int slots = (optin - static_bytes - fixed - p_bytes) / kChunkBytes;
-    if (slots > kMaxSlots) slots = kMaxSlots;
-    if (const int cap = tuning().tc_max_slots; cap >= 4 && cap < slots) slots = cap;  // testing aid: smaller rings
-    if (slots < 4) return cudaErrorInvalidConfiguration;
-    // the PV ring (refilled from L2) gets two or four slots, the QK ring the rest
-    int pv_slots = slots >= 6 ? 4 : 2;
-    if (const int v = tuning().tc_pv_slots & ~1; v >= 2 && v <= slots - 2) pv_slots = v;  // testing aid
-    const int qk_slots = slots - pv_slots;
-    const size_t smem = static_cast<size_t>(fixed) + static_cast<size_t>(slots) * kChunkBytes + p_bytes;
-    if ((e = cudaFuncSetAttribute(attn_tc_kernel<N>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    const int avail = optin - static_bytes - fixed - p_bytes;
+    // the PV ring (refilled from L2) gets six slots where four QK slots still
+    // fit beside them (streamed queries), else four or two; the QK ring the
+    // rest.  (Measured: with 80 rows six PV slots beside four QK slots beat
+    // four beside five by 6 %; eight beside two lose 50 %.)
+    int pv_slots = SQ && avail >= 4 * slot_a + 6 * kChunkBytes ? 6 : avail >= 2 * slot_a + 4 * kChunkBytes ? 4 : 2;
+    const int cap = tuning().tc_max_slots;  // testing aid: smaller rings
+    if (cap >= 4 && pv_slots > cap - 2) pv_slots = 2;
+    if (const int v = tuning().tc_pv_slots & ~1; v >= 2 && v <= kMaxSlots && avail >= 2 * slot_a + v * kChunkBytes &&
+                                                  (cap < 4 || v <= cap - 2))
+        pv_slots = v;  // testing aid
+    int qk_slots = (avail - pv_slots * kChunkBytes) / slot_a;
+    if (qk_slots > kMaxSlots) qk_slots = kMaxSlots;
+    if (cap >= 4 && qk_slots > cap - pv_slots) qk_slots = cap - pv_slots;
+    if (qk_slots < 2) return cudaErrorInvalidConfiguration;
+    const size_t smem = static_cast<size_t>(fixed) + static_cast<size_t>(qk_slots) * slot_a +
+                        static_cast<size_t>(pv_slots) * kChunkBytes + p_bytes;
+    if ((e = cudaFuncSetAttribute(attn_tc_kernel<N, SQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   static_cast<int>(smem))) != cudaSuccess)
         return e;
     TcArgs t;
@@ -1109,7 +1148,7 @@ cudaError_t launch_cfg(const AttnArgs &a, int groups, cudaStream_t st)
     t.lse_final = a.lse_final;
     t.status = a.status;
     t.wait_ns = kWaitLimitNs;
-    return launch_dependent(attn_tc_kernel<N>, dim3(groups, a.num_splits, 1), dim3(kThreads), smem, st, 1, t, mc,
+    return launch_dependent(attn_tc_kernel<N, SQ>, dim3(groups, a.num_splits, 1), dim3(kThreads), smem, st, 1, t, mc,
                             mr, mq);
 }
 
@@ -1131,12 +1170,13 @@ TcShape attn_tc_shape(int rows)
 cudaError_t launch_attn_tc(const AttnArgs &a, cudaStream_t st)
 {
     const TcShape s = attn_tc_shape(a.q_len * a.num_heads);
+    const bool sq = tuning().tc_query != 1;
     switch (s.n) {
-    case 16: return launch_cfg<16>(a, s.groups, st);
-    case 32: return launch_cfg<32>(a, s.groups, st);
-    case 48: return launch_cfg<48>(a, s.groups, st);
-    case 64: return launch_cfg<64>(a, s.groups, st);
-    case 80: return launch_cfg<80>(a, s.groups, st);
+    case 16: return sq ? launch_cfg<16, true>(a, s.groups, st) : launch_cfg<16, false>(a, s.groups, st);
+    case 32: return sq ? launch_cfg<32, true>(a, s.groups, st) : launch_cfg<32, false>(a, s.groups, st);
+    case 48: return sq ? launch_cfg<48, true>(a, s.groups, st) : launch_cfg<48, false>(a, s.groups, st);
+    case 64: return sq ? launch_cfg<64, true>(a, s.groups, st) : launch_cfg<64, false>(a, s.groups, st);
+    case 80: return sq ? launch_cfg<80, true>(a, s.groups, st) : launch_cfg<80, false>(a, s.groups, st);
     default: return cudaErrorInvalidConfiguration;
     }
 }

@@ -56,10 +56,12 @@ cudaError_t launch_attn_simt(const AttnArgs &a, cudaStream_t st);
 // CUDA-core attention; GBMLA_TC_MAX_N caps the query rows per tensor-core CTA;
 // GBMLA_TC_MAX_SLOTS caps its ring slots and GBMLA_TC_PV_SLOTS sets the share
 // of the value-product ring; GBMLA_ABSORB=persistent|gemm (absorb_path 1|2)
-// chooses the absorption kernel where both serve the shape.  0 means "not
-// set".  They change tiling only.
+// chooses the absorption kernel where both serve the shape;
+// GBMLA_TC_QUERY=resident|streamed (tc_query 1|2) keeps the queries of an
+// 80-row tensor-core CTA in shared memory or streams them with the cache
+// chunks.  0 means "not set".  They change tiling only.
 struct Tuning {
-    int attn_simt, tc_max_rows, tc_max_slots, tc_pv_slots, absorb_path;
+    int attn_simt, tc_max_rows, tc_max_slots, tc_pv_slots, absorb_path, tc_query;
 };
 const Tuning &tuning();
 void reload_tuning();

@@ -380,18 +380,24 @@ def test_tensor_core_kernel_matches_cuda_core_kernel(name, tuning):
 
 
 @pytest.mark.parametrize("env", [
-    {},                                                   # 2 x 80 rows, independent CTAs
+    {},                                                   # 2 x 80 rows, independent CTAs, streamed queries
     {"GBMLA_TC_MAX_SLOTS": "4"},                          # the smallest ring: every slot reused within a tile
     {"GBMLA_TC_MAX_N": "32", "GBMLA_TC_MAX_SLOTS": "4"},  # 5 x 32 rows
     {"GBMLA_TC_MAX_N": "48"},
     {"GBMLA_TC_MAX_N": "64"},
-], ids=["rows80", "ring4", "n32_ring4", "n48", "n64"])
+    {"GBMLA_TC_PV_SLOTS": "4"},                           # five streamed-query QK slots
+    {"GBMLA_TC_QUERY": "resident"},                       # queries resident in shared memory
+    {"GBMLA_TC_QUERY": "resident", "GBMLA_TC_MAX_SLOTS": "4"},
+    {"GBMLA_TC_QUERY": "resident", "GBMLA_TC_MAX_N": "32"},
+], ids=["rows80", "ring4", "n32_ring4", "n48", "n64", "pv4", "resident", "resident_ring4", "resident_n32"])
 @pytest.mark.parametrize("splits", [1, 3, 7])
 def test_tensor_core_kernel_shapes_and_rings(env, splits, tuning):
     """Several sequences per CTA, tail tiles of one or two pages, and rings
     smaller than a tile's chunk count (the regime where a look-ahead barrier
     wait once cleared the next sequence's rows): every query-group size and
-    ring size matches the oracle.  With 32 and 48 rows the
+    ring size matches the oracle, with the queries streamed through the
+    ring beside each cache chunk (the default) or resident in shared
+    memory.  With 32 and 48 rows the
     kernel alternates two O^T buffers between sequences and drains each after
     the next one's first tile; one split puts all five sequences in one CTA,
     so both buffers are reused and every deferred drain runs."""
