@@ -733,12 +733,12 @@ def measure_projection(args, w, dws, stream, dev, l2, peaks):
 # DRAM bytes (read + write) per attention launch from one ncu capture of the
 # kernel source with this sha256 prefix (profiles/attn_tc_<workload>.md); a
 # kernel that has changed since reports null.
-TRAFFIC_SOURCE = "0755d8d2b181673d"
+TRAFFIC_SOURCE = "d6c39a4c960d1ccd"
 TRAFFIC = {
-    "qwen05b_b16_h14_r256_t2048": 21205760,  # at 128 partitions
-    "llama3b_long_b8_h24_r512_t16k_32k": 213019136,
-    "llama1b_paged_b128_h32_r512_t128_8192": 710417152,
-    "llama1b_chunk5_b32_h32_r512_t4096": 165511424,
+    "qwen05b_b16_h14_r256_t2048": 21206016,  # at 128 partitions
+    "llama3b_long_b8_h24_r512_t16k_32k": 210286592,
+    "llama1b_paged_b128_h32_r512_t128_8192": 710535424,
+    "llama1b_chunk5_b32_h32_r512_t4096": 164428288,
 }
 
 

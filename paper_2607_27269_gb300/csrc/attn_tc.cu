@@ -44,10 +44,11 @@ constexpr int kWhole = 1 << 30;             // flag bit beside a sequence index 
 constexpr int kSoftmaxBase = 128;           // first softmax thread (after two producer and two MMA warps)
 constexpr int kThreads = kSoftmaxBase + 32 * kSoftmaxWarps;
 
-// P buffers: two (softmax of tile t overlaps PV(t-1)) where shared memory
-// allows; one for 80-row groups, whose queries leave room for little else.
+// P buffers: two, so that the softmax of tile t overlaps PV(t-1).  (With
+// streamed queries an 80-row CTA has the room; with resident ones it then
+// keeps only five ring slots.)
 template <int N>
-constexpr int kPBufs = N >= 80 ? 1 : 2;
+constexpr int kPBufs = 2;
 
 // O^T buffers in TMEM: two where they fit beside the two S^T buffers (2N + 2 x 4N
 // columns <= 512, i.e. N <= 48), so that a sequence's value products start in
@@ -1108,8 +1109,9 @@ cudaError_t launch_cfg(const AttnArgs &a, int groups, cudaStream_t st)
     const int avail = optin - static_bytes - fixed - p_bytes;
     // the PV ring (refilled from L2) gets six slots where four QK slots still
     // fit beside them (streamed queries), else four or two; the QK ring the
-    // rest.  (Measured: with 80 rows six PV slots beside four QK slots beat
-    // four beside five by 6 %; eight beside two lose 50 %.)
+    // rest.  (Measured with 80 rows, whose second P buffer leaves four QK and
+    // four PV slots: six PV slots beside three QK slots lose 16 %, two beside
+    // five 46 %.)
     int pv_slots = SQ && avail >= 4 * slot_a + 6 * kChunkBytes ? 6 : avail >= 2 * slot_a + 4 * kChunkBytes ? 4 : 2;
     const int cap = tuning().tc_max_slots;  // testing aid: smaller rings
     if (cap >= 4 && pv_slots > cap - 2) pv_slots = 2;
