@@ -46,8 +46,12 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(int batch, int
     const int sg = threadIdx.x / gsz, t = threadIdx.x % gsz;
     const int part = t % tpr, rr = t / tpr;
     const bool active = rr < rpg;  // (tpr need not divide the group)
-    const int row0 = blockIdx.x * rpg * RPT + rr;
     const bool may_be_empty = T < S;  // a partition is empty only when there are fewer tiles than partitions
+    // Row blocks blockIdx.x, + gridDim.x, ... of the unit (one per block with
+    // slot groups, whose finishing group alone goes on past the merge).
+    const int nrb = (rows + rpg * RPT - 1) / (rpg * RPT);
+    for (int rb = blockIdx.x; rb < nrb; rb += gridDim.x) {
+    const int row0 = rb * rpg * RPT + rr;
     float m[RPT], wsum[RPT], acc[RPT][8];
 #pragma unroll
     for (int r = 0; r < RPT; ++r) {
@@ -132,7 +136,7 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(int batch, int
         }
         m[0] = mx;
     }
-    if (!active) return;
+    if (!active) continue;
 #pragma unroll
     for (int r = 0; r < RPT; ++r) {
         const int row = row0 + r * rpg;
@@ -148,6 +152,7 @@ __global__ void __launch_bounds__(kCombineThreads) combine_kernel(int batch, int
         dst[1] = make_float4(acc[r][4] * inv, acc[r][5] * inv, acc[r][6] * inv, acc[r][7] * inv);
         if (lse_out && part == 0) lse_out[orow] = wsum[r] > 0.f ? m[r] + logf(wsum[r]) : -INFINITY;
     }
+    }
 }
 
 }  // namespace
@@ -160,8 +165,18 @@ cudaError_t launch_combine(int batch, int q_len, int num_heads, int rank, int ma
     const int tpr = rank / 8;
     const int rows = q_len * num_heads;
     if (batch == 0 || rows == 0) return cudaSuccess;
-    auto go = [&](auto kernel, int rows_per_block) {
-        dim3 grid((rows + rows_per_block - 1) / rows_per_block, batch);
+    // Blocks per unit.  With one row block each, the partition prologue (a
+    // reduction over every sequence's tile count) is repeated per row block;
+    // so a block of a single-group kernel takes up to four row blocks, as
+    // many as still leave four blocks per SM.  (Measured on the 128-sequence
+    // paged batch: the step 362.7 -> 358.7 us with four; with four row
+    // blocks on the 32-sequence chunk batch the combine went 9.4 -> 12.2 us.)
+    auto go = [&](auto kernel, int rows_per_block, bool looped) {
+        const int nrb = (rows + rows_per_block - 1) / rows_per_block;
+        int per = 1;
+        if (looped)
+            while (per < 4 && static_cast<int64_t>(nrb) * batch >= static_cast<int64_t>(per + 1) * 4 * 152) ++per;
+        dim3 grid((nrb + per - 1) / per, batch);
         return launch_dependent(kernel, grid, dim3(kCombineThreads), 0, st, 1, batch, q_len, num_heads, rank, max_kv,
                                 num_splits, kv_len, o_part, lse_part, o_lat, lse, groups, skip_whole ? 1 : 0);
     };
@@ -169,14 +184,14 @@ cudaError_t launch_combine(int batch, int q_len, int num_heads, int rank, int ma
     // slot groups of the smallest whole number of warps that holds a row.
     if (num_splits >= 4 * batch) {
         const int gsz = (tpr + 31) / 32 * 32;
-        if (kCombineThreads / gsz >= 8) return go(combine_kernel<1, 4, 8>, (kCombineThreads / 8) / tpr);
-        return go(combine_kernel<1, 4, 4>, (kCombineThreads / 4) / tpr);
+        if (kCombineThreads / gsz >= 8) return go(combine_kernel<1, 4, 8>, (kCombineThreads / 8) / tpr, false);
+        return go(combine_kernel<1, 4, 4>, (kCombineThreads / 4) / tpr, false);
     }
     // Few partitions per unit: rows side by side, two rows per thread once
     // that still leaves several blocks per SM
     const int rpb = kCombineThreads / tpr;
-    if (static_cast<int64_t>((rows + rpb - 1) / rpb) * batch >= 8 * 152) return go(combine_kernel<2, 2, 1>, 2 * rpb);
-    return go(combine_kernel<1, 4, 1>, rpb);
+    if (static_cast<int64_t>((rows + rpb - 1) / rpb) * batch >= 8 * 152) return go(combine_kernel<2, 2, 1>, 2 * rpb, true);
+    return go(combine_kernel<1, 4, 1>, rpb, true);
 }
 
 }  // namespace gbmla
