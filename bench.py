@@ -733,7 +733,7 @@ def measure_projection(args, w, dws, stream, dev, l2, peaks):
 # DRAM bytes (read + write) per attention launch from one ncu capture of the
 # kernel source with this sha256 prefix (profiles/attn_tc_<workload>.md); a
 # kernel that has changed since reports null.
-TRAFFIC_SOURCE = "d6c39a4c960d1ccd"
+TRAFFIC_SOURCE = "f5772acba64d9795"
 TRAFFIC = {
     "qwen05b_b16_h14_r256_t2048": 21206016,  # at 128 partitions
     "llama3b_long_b8_h24_r512_t16k_32k": 210286592,

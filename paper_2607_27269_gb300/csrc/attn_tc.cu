@@ -761,10 +761,13 @@ __global__ void __maxnreg__(128)
         // nearly size-independent time, so the loads are spread over lanes
         // and warps, each lane an independent in-order stream.  Warp 0: lane
         // s < CA refills QK-ring slot s (chunks s, s + CA, ... of the QK pass,
-        // nqc per tile: positional keys, then the latent chunks), lanes
-        // 16..16+ncc load the query boxes of each sequence.  Warp 3: lane s <
-        // CB refills PV-ring slot s (chunks s, s + CB, ... of the PV pass, ncc
-        // per tile).  The lanes of a warp poll their own barrier without
+        // nqc per tile: positional keys, then the latent chunks) -- with
+        // streamed queries the chunk's cache box(es) and then its query box
+        // (the first pass's query box waits for the next pass, after
+        // griddepcontrol.wait); with resident queries lanes 16..16+ncc load
+        // the query boxes of each sequence.  Warp 3: lane s < CB refills
+        // PV-ring slot s (chunks s, s + CB, ... of the PV pass, ncc per
+        // tile).  The lanes of a warp poll their own barrier without
         // blocking in one converged loop, and every lane whose slot is free
         // issues in the same pass.  A lane waits only on phases of its own
         // barrier, in order, so every parity test is on the next phase.
