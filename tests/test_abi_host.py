@@ -126,3 +126,31 @@ def test_acceptance_arguments_are_checked_on_the_host():
     assert L.mla_acceptance_stats(4, 100, 1, 16, 16, 100, None, None, None, None, None) == abi.MLA_ERR_INVALID_ARG
     assert L.mla_acceptance_stats(4, 100, 1, 24, 16, 104, None, None, None, None, None) == abi.MLA_ERR_INVALID_ARG
     assert L.mla_acceptance_stats(0, 100, 1, None, None, 104, None, None, None, None, None) == abi.MLA_OK
+
+
+def test_decode_step_validates_every_stage_before_the_device():
+    """mla_decode_step checks the arguments of all five stages before its
+    first launch.  With no GPU present, a bad argument of any stage -- the
+    last one's included (W_O given without `out`) -- comes back as
+    MLA_ERR_INVALID_ARG, while a call whose arguments are all valid gets as
+    far as the device and fails there; an empty batch is a no-op."""
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present: the all-valid call would launch on stand-in pointers")
+    L = abi.lib()
+    d = _dims(hidden=256).c()
+    c = abi.MlaCache(0x1000, 0x2000, 512, 64, 512 * 64, 64 * 64, None, 0, 0, 0, 64)
+    A = 0x10000  # 16-byte aligned stand-in for every buffer (never dereferenced: no device)
+
+    def step(batch=2, q_len=1, c_new=A, kr_new=A, start_pos=A, max_kv=64, splits=4, q_abs=A, o_lat=A, out=A):
+        return L.mla_decode_step(ctypes.byref(d), ctypes.byref(c), batch, q_len, c_new, kr_new, start_pos, A, A, A,
+                                 max_kv, A, A, A, splits, q_abs, A, A, o_lat, A, A, out, None)
+
+    assert step() == abi.MLA_ERR_CUDA
+    assert step(batch=0) == abi.MLA_OK
+    assert step(out=None) == abi.MLA_ERR_INVALID_ARG        # out_proj, the fifth stage
+    assert step(o_lat=A + 4) == abi.MLA_ERR_INVALID_ARG     # combine / out_proj
+    assert step(q_abs=None) == abi.MLA_ERR_INVALID_ARG      # absorption / attention
+    assert step(splits=-1) == abi.MLA_ERR_INVALID_ARG       # attention
+    assert step(c_new=A + 2) == abi.MLA_ERR_INVALID_ARG     # append, the first stage
+    assert step(q_len=4, max_kv=2) == abi.MLA_ERR_INVALID_ARG
